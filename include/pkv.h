@@ -1,0 +1,229 @@
+/*
+ * pkv.h -- C ABI of the prefix-cached paged-attention library (libpkv.so).
+ *
+ * The library implements the data-parallel hot path of the "Reuse plane" of
+ * the compliance serving stack of arXiv 2605.11232 (Fig. 1): attention over a
+ * KV cache kept in fixed-size physical blocks addressed through per-request
+ * block tables (PagedAttention, Sec. 2 and Sec. 5.4), whose leading blocks can
+ * be a policy/schema prefix shared by many requests and stored once
+ * (Automatic Prefix Caching, Sec. 2 and Sec. 5.4; the design rule at the end
+ * of Sec. 3 that shared prefixes are not recomputed).
+ *
+ * Conventions for every call
+ *  - All device buffers are owned by the caller.  The library keeps host
+ *    metadata (free list, reference counts, TMA descriptors) and one small
+ *    device error word per pool, allocated by kv_pool_create.
+ *  - "device" pointers are CUDA global-memory addresses on the pool's device;
+ *    "host" pointers are ordinary CPU memory.  Device buffers must be 16-byte
+ *    aligned and contiguous in the stated layout.
+ *  - Kernels are enqueued on `stream` (a cudaStream_t; NULL is the legacy
+ *    default stream) and return before they run.  Argument errors are found
+ *    on the host and returned before anything is enqueued; errors seen by a
+ *    kernel (an out-of-range slot or block id, a bounded wait that ran out)
+ *    are latched in the pool's device error word and reported by
+ *    pkv_check_device_errors.
+ *  - Every call returns PKV_OK (0) or a negative pkv_status; pkv_last_error()
+ *    then gives a message (per thread).  No C++ exception crosses the ABI.
+ *  - Element type: bf16 only.  Block size: 16 tokens.  Head dim: 64 or 128.
+ *    num_q_heads must be a multiple of num_kv_heads; q heads h belong to kv
+ *    head h / (num_q_heads / num_kv_heads) (contiguous GQA grouping).
+ *  - A pool handle is not thread-safe; calls on one handle must not overlap.
+ */
+#ifndef PKV_H
+#define PKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct pkv_pool *pkv_pool_t;
+typedef void *pkv_stream_t; /* a cudaStream_t */
+
+typedef enum {
+    PKV_OK = 0,
+    PKV_ERR_INVALID_ARG = -1,        /* null pointer, bad size or layout        */
+    PKV_ERR_OUT_OF_BLOCKS = -2,      /* free list cannot satisfy an allocation   */
+    PKV_ERR_REFCOUNT = -3,           /* release of a free block, bad id          */
+    PKV_ERR_SHARED_BLOCK_WRITE = -4, /* a slot lies in a block with refcount > 1 */
+    PKV_ERR_CUDA = -5,               /* a CUDA runtime/driver call failed        */
+    PKV_ERR_UNSUPPORTED = -6,        /* shape outside what the kernels handle    */
+    PKV_ERR_WORKSPACE = -7,          /* workspace missing or too small           */
+    PKV_ERR_DEVICE_TIMEOUT = -8,     /* a bounded device wait ran out            */
+    PKV_ERR_DEVICE_BOUNDS = -9       /* a kernel met an out-of-range slot/block  */
+} pkv_status;
+
+enum { PKV_DTYPE_BF16 = 1 };
+
+/* Physical block pool.  K and V caches are separate device arrays of
+ * num_blocks * num_kv_heads * block_size * head_dim bf16 values laid out as
+ * [num_blocks][num_kv_heads][block_size][head_dim]: the 16 tokens of one
+ * (block, kv head) pair are one contiguous tile (4 KiB at head_dim 128). */
+typedef struct {
+    int32_t num_blocks;      /* > 0                                              */
+    int32_t block_size;      /* must be 16                                       */
+    int32_t num_kv_heads;    /* > 0                                              */
+    int32_t head_dim;        /* 64 or 128                                        */
+    int32_t dtype;           /* PKV_DTYPE_BF16                                   */
+    int32_t reserved;        /* 0                                                */
+    uint64_t placement_seed; /* 0: blocks are handed out as 0,1,2,...; otherwise
+                                the initial free list is a permutation drawn
+                                from this seed (splitmix64 + Fisher-Yates)      */
+} pkv_pool_desc;
+
+/* Shared-prefix groups of a decode batch (APC, Sec. 5.4).  Group g owns the
+ * first group_blocks[g] table entries of each of its member requests: those
+ * entries are the same physical blocks for every member, hold full 16-token
+ * blocks of the shared prefix, and are never written.  With groups, decode
+ * reads each shared block once per group and kv head instead of once per
+ * request.  All arrays are device arrays. */
+typedef struct {
+    int32_t num_groups;        /* G >= 0; 0 means no sharing information         */
+    int32_t max_group_blocks;  /* host upper bound on group_blocks[g]            */
+    int32_t max_group_members; /* host upper bound on members of one group       */
+    int32_t reserved;          /* 0                                              */
+    const int32_t *group_start;  /* [G+1] CSR offsets into member_req            */
+    const int32_t *member_req;   /* [group_start[G]] request indices, by group   */
+    const int32_t *group_blocks; /* [G] shared leading blocks of group g (>= 0)  */
+    const int32_t *group_of_req; /* [num_requests] group of request r, -1: none  */
+} pkv_prefix_groups;
+
+/* ---- a1: pool and reference counts (host) ------------------------------- */
+
+/* Create a pool over caller-owned device caches (Sec. 2, Sec. 5.4: paged KV
+ * memory).  k_cache/v_cache: device, layout above; both NULL gives a
+ * metadata-only pool (allocation calls work, kernel calls fail with
+ * PKV_ERR_INVALID_ARG).  On success *out owns host metadata and a 4-byte device
+ * error word; free it with kv_pool_destroy.  Errors: INVALID_ARG, UNSUPPORTED
+ * (block_size != 16, head_dim not 64/128, dtype not bf16), CUDA. */
+int kv_pool_create(const pkv_pool_desc *desc, void *k_cache, void *v_cache, pkv_pool_t *out);
+
+/* Free the host metadata and the error word (not the caches).  NULL is a no-op. */
+int kv_pool_destroy(pkv_pool_t pool);
+
+/* Take n free blocks; their ids go to ids_out (host, n entries), each with
+ * reference count 1.  All or nothing: OUT_OF_BLOCKS leaves the pool as it was. */
+int kv_pool_alloc(pkv_pool_t pool, int32_t n, int32_t *ids_out);
+
+/* Add one reference to each listed block (host ids): a request that reuses a
+ * cached prefix holds its blocks this way (APC, Sec. 5.4).  REFCOUNT if an id
+ * is out of range or free; nothing changes on error. */
+int kv_pool_retain(pkv_pool_t pool, const int32_t *ids, int32_t n);
+
+/* Drop one reference from each listed block (host ids); a block whose count
+ * reaches 0 returns to the free list.  REFCOUNT on a free or out-of-range id,
+ * or on an id listed more times than it has references; nothing changes on
+ * error. */
+int kv_pool_release(pkv_pool_t pool, const int32_t *ids, int32_t n);
+
+/* Reference count of one block (0 = free).  INVALID_ARG on a bad id. */
+int kv_pool_refcount(pkv_pool_t pool, int32_t id, int32_t *out);
+
+/* Number of free blocks. */
+int kv_pool_num_free(pkv_pool_t pool, int32_t *out);
+
+/* One request's block-table row (a1 + a2): retain the n_prefix shared prefix
+ * blocks `prefix_ids` (host; may be NULL when n_prefix is 0), allocate
+ * n_blocks - n_prefix private blocks, and write the row to row_out (host,
+ * n_blocks entries): prefix ids first, then the new private ids in order.
+ * All or nothing. */
+int kv_pool_alloc_sequence(pkv_pool_t pool, const int32_t *prefix_ids, int32_t n_prefix,
+                           int32_t n_blocks, int32_t *row_out);
+
+/* ---- a2: slot mapping (host) -------------------------------------------- */
+
+/* Slot of every new token (PagedAttention addressing, Sec. 2): new token i of
+ * request r is at position p = context_lens[r] - new_lens[r] + i and goes to
+ * slot block_table[r][p / 16] * 16 + p % 16.  Tokens are numbered request
+ * after request.  All arrays are host arrays; block_table is [R][max_blocks]
+ * row-major; slots_out has sum(new_lens) entries.  With a pool (non-NULL),
+ * every target block must be allocated and unshared: a slot in a block with
+ * reference count > 1 returns SHARED_BLOCK_WRITE (shared prefix blocks are
+ * immutable), a free or out-of-range block REFCOUNT.  pool may be NULL (no
+ * ownership checks). */
+int kv_slot_mapping(pkv_pool_t pool, const int32_t *block_table, int32_t max_blocks,
+                    const int32_t *context_lens, const int32_t *new_lens, int32_t num_requests,
+                    int64_t *slots_out);
+
+/* ---- a3: cache write (device) ------------------------------------------- */
+
+/* Scatter new-token keys and values into their slots (bit-exact copy).
+ * k_new, v_new: device bf16 [num_tokens][num_kv_heads][head_dim].
+ * slot_mapping: device int64 [num_tokens]; slot s goes to block s / 16, offset
+ * s % 16; s < 0 skips the token; s >= num_blocks * 16 is skipped and latches
+ * DEVICE_BOUNDS.  Two tokens with the same slot: undefined which one lands.
+ * num_tokens == 0 is a no-op. */
+int kv_cache_write(pkv_pool_t pool, const void *k_new, const void *v_new,
+                   const int64_t *slot_mapping, int32_t num_tokens, pkv_stream_t stream);
+
+/* ---- a4: suffix prefill over cached context (device) -------------------- */
+
+/* Attention of the new (suffix or chunk) tokens of each request: new token i
+ * of request r, at position p = context_lens[r] - n_r + i with
+ * n_r = cu_seqlens_q[r+1] - cu_seqlens_q[r], attends to every cached key of
+ * the request (shared prefix included) and causally to the new keys, i.e. to
+ * positions 0..p, read through the block table (Sec. 5.4: the cached prefix
+ * is reused, only the suffix is computed).  The new tokens' K/V must already
+ * be in the cache (kv_cache_write).
+ *  q, out: device bf16 [T][num_q_heads][head_dim], T = cu_seqlens_q[R].
+ *  lse: device fp32 [T][num_q_heads] natural-log log-sum-exp, or NULL.
+ *  cu_seqlens_q: device int32 [R+1], non-decreasing from 0.
+ *  context_lens: device int32 [R], context_lens[r] >= n_r (includes them).
+ *  block_table: device int32 [R][max_blocks]; entries past ceil(L/16) unread.
+ *  max_seqlen_q: host upper bound on n_r (sizes the grid); requests with
+ *  n_r = 0 are skipped.
+ *  scale: softmax scale (normally 1/sqrt(head_dim)).
+ * Errors: INVALID_ARG, UNSUPPORTED (num_q_heads / num_kv_heads > 128), CUDA. */
+int paged_attn_prefill(pkv_pool_t pool, const void *q, void *out, float *lse,
+                       const int32_t *cu_seqlens_q, const int32_t *context_lens,
+                       const int32_t *block_table, int32_t max_blocks, int32_t num_requests,
+                       int32_t max_seqlen_q, int32_t num_q_heads, float scale,
+                       pkv_stream_t stream);
+
+/* ---- a5-a7: decode (device) ---------------------------------------------- */
+
+/* Bytes of workspace paged_attn_decode needs for these shapes (host call).
+ * groups may be NULL. */
+int paged_attn_decode_workspace_size(pkv_pool_t pool, int32_t num_requests,
+                                     int32_t num_q_heads, int32_t max_blocks,
+                                     const pkv_prefix_groups *groups, size_t *bytes_out);
+
+/* One query token per request attends to all context_lens[r] keys of its
+ * block list (the decode step of Sec. 5.3's short structured outputs).  The
+ * query token's own K/V must already be in the cache.  Keys are split into
+ * ranges processed in parallel, each producing an unnormalised partial output
+ * with its running max and sum; a combine pass merges them by log-sum-exp
+ * weights.  With groups, the shared prefix blocks of each group are processed
+ * once per group for all member requests.
+ *  q, out: device bf16 [R][num_q_heads][head_dim].
+ *  lse: device fp32 [R][num_q_heads] (natural log) or NULL.
+ *  context_lens: device int32 [R], each >= 1 (and > 16 * shared blocks).
+ *  block_table: device int32 [R][max_blocks].
+ *  groups: NULL, or a descriptor as above.
+ *  workspace: device scratch of at least paged_attn_decode_workspace_size()
+ *  bytes, 256-byte aligned; its contents need no initialisation and are
+ *  clobbered.
+ * Errors: INVALID_ARG, UNSUPPORTED (group size g > 8), WORKSPACE, CUDA. */
+int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
+                      const int32_t *context_lens, const int32_t *block_table,
+                      int32_t max_blocks, int32_t num_requests, int32_t num_q_heads,
+                      float scale, const pkv_prefix_groups *groups, void *workspace,
+                      size_t workspace_bytes, pkv_stream_t stream);
+
+/* ---- errors --------------------------------------------------------------- */
+
+/* Synchronise `stream`, then read and clear the pool's device error word.
+ * *code_out gets PKV_OK or the first latched device status (DEVICE_BOUNDS,
+ * DEVICE_TIMEOUT).  The return value reports failures of the call itself. */
+int pkv_check_device_errors(pkv_pool_t pool, pkv_stream_t stream, int32_t *code_out);
+
+/* Message of the last failing call on this thread ("" if none). */
+const char *pkv_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PKV_H */

@@ -1,0 +1,461 @@
+// decode.cu -- split-KV paged decode attention (one query token per request).
+//
+// The decode step of the paper's short structured outputs (Sec. 5.3) reads
+// each request's whole block list (PagedAttention, Sec. 2 / Sec. 5.4) for one
+// query token.  With GQA the g q-heads of a kv head share every K/V row, so
+// the arithmetic intensity is ~g FLOP per byte: HBM-bound once the dot
+// products run on tensor cores.
+//
+// Work split ("pieces").  The private blocks of all (request, kv head) pairs
+// form one stream of W blocks, segment (r, h) after segment.  Warp w of the
+// persistent grid takes blocks [w*per, (w+1)*per) of that stream, so every
+// warp moves the same number of bytes whatever the length mix; a warp that
+// crosses a segment boundary emits one unnormalised partial (O, m, l) per
+// segment it touches.  The combine kernel merges a head's partials with
+// log-sum-exp weights.
+//
+// Inner loop (one 16-token block per step, per warp):
+//   S^T[16 keys x 8 heads] = K_blk[16 x d] . Q^T[d x 8]   (mma m16n8k16, A = K)
+//   online softmax per head column (shuffles across the 8 row groups)
+//   O^T[d x 8] += V_blk^T[d x 16] . P^T[16 x 8]           (A = V^T, B = P^T)
+// K and V are read with 16-byte loads straight into registers in the order
+// the mma fragments need: the head dimension is a contraction index for
+// Q.K and the key index one for P.V, so both may be permuted freely as long
+// as both operands use the same permutation.  The S^T accumulator becomes the
+// P^T operand through one movmatrix transpose per 8x8 quadrant; the key order
+// sigma() of the QK^T rows is chosen so that the transposed fragments land on
+// exactly the keys each thread loaded for P.V.
+#include <math.h>
+
+#include "pkv_device.cuh"
+#include "pkv_internal.h"
+
+namespace pkv {
+
+namespace {
+
+constexpr int kWarps = 8;
+constexpr int kThreads = kWarps * 32;
+constexpr int kMaxRequestsPlan = 16384;
+
+__device__ __forceinline__ uint32_t reg_of(const uint4 &v, int i) {
+    return i == 0 ? v.x : (i == 1 ? v.y : (i == 2 ? v.z : v.w));
+}
+
+// Physical key (row of the 16-token block) behind logical QK^T row r (0..7);
+// row r + 8 is sigma(r) + 2.
+__device__ __forceinline__ int sigma(int r) { return 2 * r - (r & 1); }
+
+template <int D>
+struct BlockRegs {
+    uint4 ka[D / 32];   // K[sigma(r)    ][chunk 4j+q]
+    uint4 kb[D / 32];   // K[sigma(r) + 2][chunk 4j+q]
+    uint4 va[4];        // V[4q+s][chunk r]       (d 8r..8r+7)
+    uint4 vb[D == 128 ? 4 : 1];   // V[4q+s][chunk 8+r] (d 64+8r..), d = 128 only
+};
+
+template <int D>
+__device__ __forceinline__ void load_block(BlockRegs<D> &b, const uint16_t *kt,
+                                           const uint16_t *vt, int lr, int lq) {
+    const int s0 = sigma(lr);
+#pragma unroll
+    for (int j = 0; j < D / 32; ++j) {
+        b.ka[j] = ldg_stream(kt + s0 * D + (4 * j + lq) * 8);
+        b.kb[j] = ldg_stream(kt + (s0 + 2) * D + (4 * j + lq) * 8);
+    }
+#pragma unroll
+    for (int s = 0; s < 4; ++s) {
+        b.va[s] = ldg_stream(vt + (4 * lq + s) * D + lr * 8);
+        if constexpr (D == 128) b.vb[s] = ldg_stream(vt + (4 * lq + s) * D + (8 + lr) * 8);
+    }
+}
+
+// Running state of one warp over one piece.  Thread (lr = lane/4, lq = lane%4)
+// holds heads 2lq, 2lq+1: m, l (thread-partial sum) and O^T fragments.
+template <int D>
+struct SoftmaxState {
+    float m[2];
+    float l[2];
+    float o[D / 16][4];
+};
+
+template <int D>
+__device__ __forceinline__ void attend_block(SoftmaxState<D> &st, BlockRegs<D> &b,
+                                             const uint32_t (&qf)[D / 32][4], int lr, int lq,
+                                             int valid_keys, float scale_log2) {
+    // S^T = K . Q^T
+    float sacc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int s = 0; s < D / 16; ++s) {
+        const int j = s >> 1, e = s & 1;
+        mma_bf16_16816(sacc, reg_of(b.ka[j], 2 * e), reg_of(b.kb[j], 2 * e),
+                       reg_of(b.ka[j], 2 * e + 1), reg_of(b.kb[j], 2 * e + 1), qf[j][2 * e],
+                       qf[j][2 * e + 1]);
+    }
+    const int key0 = sigma(lr), key1 = key0 + 2;
+    const bool ok0 = key0 < valid_keys, ok1 = key1 < valid_keys;
+    float s00 = ok0 ? sacc[0] * scale_log2 : -INFINITY;   // key0, head 2lq
+    float s01 = ok0 ? sacc[1] * scale_log2 : -INFINITY;   // key0, head 2lq+1
+    float s10 = ok1 ? sacc[2] * scale_log2 : -INFINITY;   // key1, head 2lq
+    float s11 = ok1 ? sacc[3] * scale_log2 : -INFINITY;   // key1, head 2lq+1
+    float mx0 = fmaxf(s00, s10), mx1 = fmaxf(s01, s11);
+#pragma unroll
+    for (int off = 4; off < 32; off <<= 1) {
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, off));
+    }
+    const float mn0 = fmaxf(st.m[0], mx0), mn1 = fmaxf(st.m[1], mx1);
+    // mn is finite: every processed block has at least one valid key.
+    const float a0 = fast_exp2(st.m[0] - mn0), a1 = fast_exp2(st.m[1] - mn1);
+    st.m[0] = mn0;
+    st.m[1] = mn1;
+    const float p00 = fast_exp2(s00 - mn0), p10 = fast_exp2(s10 - mn0);
+    const float p01 = fast_exp2(s01 - mn1), p11 = fast_exp2(s11 - mn1);
+    st.l[0] = st.l[0] * a0 + (p00 + p10);
+    st.l[1] = st.l[1] * a1 + (p01 + p11);
+#pragma unroll
+    for (int i = 0; i < D / 16; ++i) {
+        st.o[i][0] *= a0;
+        st.o[i][2] *= a0;
+        st.o[i][1] *= a1;
+        st.o[i][3] *= a1;
+    }
+    // P^T fragments: transpose the two 8x8 quadrants of P^T(key, head).
+    const uint32_t t0 = movmatrix_trans(pack_bf16x2(p00, p01));
+    const uint32_t t1 = movmatrix_trans(pack_bf16x2(p10, p11));
+    // Masked keys carry p = 0, but 0 * NaN would poison O: zero their V rows.
+#pragma unroll
+    for (int s = 0; s < 4; ++s) {
+        if (4 * lq + s >= valid_keys) {
+            b.va[s] = make_uint4(0, 0, 0, 0);
+            if constexpr (D == 128) b.vb[s] = make_uint4(0, 0, 0, 0);
+        }
+    }
+    // O^T += V^T . P^T, one 16-row tile of the head dim per mma.
+#pragma unroll
+    for (int i = 0; i < D / 16; ++i) {
+        const uint4 *src = (i < 4) ? b.va : b.vb;
+        const int w = i & 3;
+        const uint32_t x0 = reg_of(src[0], w), x1 = reg_of(src[1], w);
+        const uint32_t x2 = reg_of(src[2], w), x3 = reg_of(src[3], w);
+        mma_bf16_16816(st.o[i], __byte_perm(x0, x1, 0x5410), __byte_perm(x0, x1, 0x7632),
+                       __byte_perm(x2, x3, 0x5410), __byte_perm(x2, x3, 0x7632), t0, t1);
+    }
+}
+
+// Block-wide plan: P[r] = sum of the private block counts of requests < r,
+// P[R] = their total; *max_n_out = the largest count.
+__device__ void build_plan(int32_t *P, int32_t R, const int32_t *__restrict__ context_lens,
+                           const int32_t *__restrict__ group_of_req,
+                           const int32_t *__restrict__ group_blocks, int32_t num_groups,
+                           int32_t max_blocks, int32_t *max_n_out, int *err) {
+    __shared__ int32_t warp_tot[kWarps];
+    __shared__ int32_t warp_max[kWarps];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int per_thread = (R + kThreads - 1) / kThreads;
+    const int r0 = min(R, tid * per_thread), r1 = min(R, r0 + per_thread);
+    int32_t run = 0, mx = 0;
+    for (int r = r0; r < r1; ++r) {
+        const int32_t L = __ldg(context_lens + r);
+        int32_t nblk = (L + 15) >> 4;
+        if (nblk > max_blocks) {   // context longer than the table row
+            latch_error(err, kDevBounds);
+            nblk = max_blocks;
+        }
+        int32_t sh = 0;
+        if (num_groups > 0) {
+            const int32_t gi = __ldg(group_of_req + r);
+            if (gi >= 0 && gi < num_groups) sh = __ldg(group_blocks + gi);
+        }
+        int32_t n = nblk - sh;
+        if (L < 1 || n < 1 || sh < 0) {   // decode needs a private tail block holding the query
+            latch_error(err, kDevBounds);
+            n = 1;
+            sh = 0;
+        }
+        P[r] = n;   // the count for now; this thread alone touches P[r0..r1)
+        run += n;
+        mx = max(mx, n);
+    }
+    int32_t incl = run;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        const int32_t v = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off) incl += v;
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    if (lane == 31) warp_tot[warp] = incl;
+    if (lane == 0) warp_max[warp] = mx;
+    __syncthreads();
+    int32_t base = 0, total = 0, gmax = 0;
+    for (int w = 0; w < kWarps; ++w) {
+        if (w < warp) base += warp_tot[w];
+        total += warp_tot[w];
+        gmax = max(gmax, warp_max[w]);
+    }
+    int32_t acc = base + incl - run;   // exclusive prefix at r0
+    for (int r = r0; r < r1; ++r) {
+        const int32_t n = P[r];
+        P[r] = acc;
+        acc += n;
+    }
+    if (tid == 0) {
+        P[R] = total;
+        *max_n_out = gmax;
+    }
+    __syncthreads();
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1) decode_split_kernel(DecodeArgs a, DecodeLayout lay,
+                                                                  int32_t num_blocks_pool) {
+    extern __shared__ int32_t P[];   // [R + 1]
+    __shared__ int32_t s_max_n;
+    const int32_t R = lay.R, Hkv = lay.Hkv, Hq = lay.Hq, g = lay.g;
+    build_plan(P, R, a.context_lens, a.group_of_req, a.group_blocks, a.num_groups, a.max_blocks,
+               &s_max_n, a.err);
+    const int64_t W = (int64_t)Hkv * P[R];
+    const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+    int64_t per = (W + nwarps - 1) / nwarps;
+    const int64_t need = (s_max_n - 1 + kMaxPrivateParts - 3) / (kMaxPrivateParts - 2);
+    if (per < need) per = need;
+    if (per < kMinBlocksPerPiece) per = kMinBlocksPerPiece;
+
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int lr = lane >> 2, lq = lane & 3;
+    const int64_t w = (int64_t)blockIdx.x * kWarps + warp;
+    int64_t x = w * per;
+    const int64_t x_end = min(x + per, W);
+
+    const uint16_t *q = static_cast<const uint16_t *>(a.q);
+    const uint16_t *kc = static_cast<const uint16_t *>(a.k_cache);
+    const uint16_t *vc = static_cast<const uint16_t *>(a.v_cache);
+    float *o_part = reinterpret_cast<float *>(static_cast<char *>(a.ws) + lay.off_o);
+    float2 *ml_part = reinterpret_cast<float2 *>(static_cast<char *>(a.ws) + lay.off_ml);
+    int32_t *nparts = reinterpret_cast<int32_t *>(static_cast<char *>(a.ws) + lay.off_nparts);
+
+    while (x < x_end) {
+        // segment containing x: request r (largest r with P[r] <= x / Hkv), head h
+        const int64_t xr = x / Hkv;
+        int lo = 0, hi = R - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (P[mid] <= xr) lo = mid; else hi = mid - 1;
+        }
+        const int r = lo;
+        const int32_t n = P[r + 1] - P[r];
+        const int64_t seg_base = (int64_t)Hkv * P[r];
+        const int h = (int)((x - seg_base) / n);
+        const int64_t seg_off = seg_base + (int64_t)h * n;
+        const int64_t piece_end = min(x_end, seg_off + n);
+        const int b_lo = (int)(x - seg_off), b_hi = (int)(piece_end - seg_off);
+        const int part = (int)(x / per - seg_off / per);
+
+        const int32_t L = __ldg(a.context_lens + r);
+        // shared leading blocks: the plan's private count n ends at the last block
+        const int32_t nblk = min((L + 15) >> 4, a.max_blocks);
+        const int32_t sh = max(nblk - n, 0);
+        const int32_t *trow = a.block_table + (int64_t)r * a.max_blocks;
+
+        // Q fragments of the g heads of kv head h (head lr of the group)
+        uint32_t qf[D / 32][4];
+        {
+            const bool hv = lr < g;
+            const uint16_t *qrow = q + ((int64_t)r * Hq + h * g + (hv ? lr : 0)) * D;
+#pragma unroll
+            for (int j = 0; j < D / 32; ++j) {
+                uint4 v = hv ? ldg16(qrow + (4 * j + lq) * 8) : make_uint4(0, 0, 0, 0);
+                qf[j][0] = v.x; qf[j][1] = v.y; qf[j][2] = v.z; qf[j][3] = v.w;
+            }
+        }
+        SoftmaxState<D> st;
+        st.m[0] = st.m[1] = -INFINITY;
+        st.l[0] = st.l[1] = 0.f;
+#pragma unroll
+        for (int i = 0; i < D / 16; ++i) st.o[i][0] = st.o[i][1] = st.o[i][2] = st.o[i][3] = 0.f;
+
+        // block ids of this piece, 32 at a time, one per lane
+        int win_base = b_lo;
+        int32_t my_phys = 0;
+        auto refresh = [&](int base) {
+            win_base = base;
+            const int bi = sh + base + lane;
+            int32_t p = (base + lane < b_hi) ? __ldg(trow + bi) : 0;
+            if (p < 0 || p >= num_blocks_pool) {
+                if (base + lane < b_hi) latch_error(a.err, kDevBounds);
+                p = 0;
+            }
+            my_phys = p;
+        };
+        refresh(b_lo);
+        auto tile_of = [&](int b, const uint16_t *base) {
+            if (b - win_base >= 32) refresh(b);
+            const int32_t phys = __shfl_sync(0xffffffffu, my_phys, b - win_base);
+            return base + ((int64_t)phys * Hkv + h) * 16 * D;
+        };
+        auto valid_of = [&](int b) {
+            const int pos0 = (sh + b) * 16;
+            return min(16, L - pos0);
+        };
+
+        BlockRegs<D> b0, b1;
+        load_block<D>(b0, tile_of(b_lo, kc), tile_of(b_lo, vc), lr, lq);
+        for (int b = b_lo; b < b_hi; b += 2) {
+            if (b + 1 < b_hi) load_block<D>(b1, tile_of(b + 1, kc), tile_of(b + 1, vc), lr, lq);
+            attend_block<D>(st, b0, qf, lr, lq, valid_of(b), a.scale_log2);
+            if (b + 1 >= b_hi) break;
+            if (b + 2 < b_hi) load_block<D>(b0, tile_of(b + 2, kc), tile_of(b + 2, vc), lr, lq);
+            attend_block<D>(st, b1, qf, lr, lq, valid_of(b + 1), a.scale_log2);
+        }
+
+        // row-group reduction of the thread-partial sums
+#pragma unroll
+        for (int off = 4; off < 32; off <<= 1) {
+            st.l[0] += __shfl_xor_sync(0xffffffffu, st.l[0], off);
+            st.l[1] += __shfl_xor_sync(0xffffffffu, st.l[1], off);
+        }
+        const int slot_part = lay.prefix_parts + part;
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+            const int hd = 2 * lq + c;
+            if (hd < g) {
+                const int64_t slot = ((int64_t)r * Hq + h * g + hd) * lay.parts_per_head + slot_part;
+                float *dst = o_part + slot * D;
+#pragma unroll
+                for (int half = 0; half < D / 64; ++half) {
+                    const int i0 = half * 4;
+                    float4 v0 = make_float4(st.o[i0][c], st.o[i0][2 + c], st.o[i0 + 1][c],
+                                            st.o[i0 + 1][2 + c]);
+                    float4 v1 = make_float4(st.o[i0 + 2][c], st.o[i0 + 2][2 + c],
+                                            st.o[i0 + 3][c], st.o[i0 + 3][2 + c]);
+                    float4 *p4 = reinterpret_cast<float4 *>(dst + half * 64 + lr * 8);
+                    p4[0] = v0;
+                    p4[1] = v1;
+                }
+                if (lr == 0) ml_part[slot] = make_float2(st.m[c], st.l[c]);
+            }
+        }
+        if (x == seg_off && lane == 0) {
+            nparts[(int64_t)r * Hkv + h] = (int32_t)((seg_off + n - 1) / per - seg_off / per + 1);
+        }
+        x = piece_end;
+    }
+}
+
+// Merge the partials of each (request, q head) with log-sum-exp weights.
+template <int D>
+__global__ void __launch_bounds__(256) decode_combine_kernel(DecodeArgs a, DecodeLayout lay) {
+    const int lane = threadIdx.x & 31;
+    const int64_t item = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
+    if (item >= (int64_t)lay.R * lay.Hq) return;
+    const int r = (int)(item / lay.Hq), hq = (int)(item % lay.Hq);
+    const int h = hq / lay.g;
+    const float *o_part = reinterpret_cast<const float *>(static_cast<const char *>(a.ws) + lay.off_o);
+    const float2 *ml_part =
+        reinterpret_cast<const float2 *>(static_cast<const char *>(a.ws) + lay.off_ml);
+    const int32_t *nparts =
+        reinterpret_cast<const int32_t *>(static_cast<const char *>(a.ws) + lay.off_nparts);
+    int n_pre = 0;
+    if (a.num_groups > 0) {
+        const int32_t gi = __ldg(a.group_of_req + r);
+        if (gi >= 0 && gi < a.num_groups) {
+            const int32_t gb = __ldg(a.group_blocks + gi);
+            n_pre = (gb + lay.prefix_blocks_per_part - 1) / lay.prefix_blocks_per_part;
+            n_pre = min(n_pre, lay.prefix_parts);
+        }
+    }
+    const int n_priv = min(max(__ldg(nparts + (int64_t)r * lay.Hkv + h), 0), kMaxPrivateParts);
+    const int total = n_pre + n_priv;
+    const int64_t slot0 = item * lay.parts_per_head;
+    auto part_slot = [&](int k) {
+        return slot0 + (k < n_pre ? k : lay.prefix_parts + (k - n_pre));
+    };
+    // each lane holds up to two parts' (m, l)
+    float m_a = -INFINITY, l_a = 0.f, m_b = -INFINITY, l_b = 0.f;
+    if (lane < total) { float2 v = ml_part[part_slot(lane)]; m_a = v.x; l_a = v.y; }
+    if (lane + 32 < total) { float2 v = ml_part[part_slot(lane + 32)]; m_b = v.x; l_b = v.y; }
+    float mx = fmaxf(m_a, m_b);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    const float w_a = (lane < total) ? fast_exp2(m_a - mx) : 0.f;
+    const float w_b = (lane + 32 < total) ? fast_exp2(m_b - mx) : 0.f;
+    float den = w_a * l_a + w_b * l_b;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) den += __shfl_xor_sync(0xffffffffu, den, off);
+    const float inv = 1.f / den;
+    constexpr int E = D / 32;   // elements per lane
+    float acc[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) acc[e] = 0.f;
+    for (int k = 0; k < total; ++k) {
+        const float wk = __shfl_sync(0xffffffffu, k < 32 ? w_a : w_b, k & 31);
+        const float *src = o_part + part_slot(k) * D + lane * E;
+        if constexpr (E == 4) {
+            const float4 v = *reinterpret_cast<const float4 *>(src);
+            acc[0] += wk * v.x; acc[1] += wk * v.y; acc[2] += wk * v.z; acc[3] += wk * v.w;
+        } else {
+            const float2 v = *reinterpret_cast<const float2 *>(src);
+            acc[0] += wk * v.x; acc[1] += wk * v.y;
+        }
+    }
+    uint16_t *out = static_cast<uint16_t *>(a.out) + item * D + lane * E;
+    if constexpr (E == 4) {
+        uint2 pk = make_uint2(pack_bf16x2(acc[0] * inv, acc[1] * inv),
+                              pack_bf16x2(acc[2] * inv, acc[3] * inv));
+        *reinterpret_cast<uint2 *>(out) = pk;
+    } else {
+        *reinterpret_cast<uint32_t *>(out) = pack_bf16x2(acc[0] * inv, acc[1] * inv);
+    }
+    if (a.lse && lane == 0) a.lse[item] = (mx + __log2f(den)) * 0.69314718055994530942f;
+}
+
+}  // namespace
+
+DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_t max_blocks,
+                           int32_t num_groups, int32_t max_group_blocks) {
+    DecodeLayout L{};
+    L.R = R; L.Hq = Hq; L.Hkv = Hkv; L.d = d; L.g = Hq / Hkv;
+    L.prefix_blocks_per_part = 64;
+    L.prefix_parts = 0;
+    if (num_groups > 0 && max_group_blocks > 0)
+        L.prefix_parts = (max_group_blocks + L.prefix_blocks_per_part - 1) / L.prefix_blocks_per_part;
+    L.parts_per_head = L.prefix_parts + kMaxPrivateParts;
+    const size_t slots = (size_t)R * Hq * L.parts_per_head;
+    auto up = [](size_t x) { return (x + 255) & ~(size_t)255; };
+    L.off_o = 0;
+    L.off_ml = up(slots * d * sizeof(float));
+    L.off_nparts = L.off_ml + up(slots * sizeof(float2));
+    L.total = L.off_nparts + up((size_t)R * Hkv * sizeof(int32_t));
+    (void)max_blocks;
+    return L;
+}
+
+template <int D>
+static cudaError_t launch_decode_t(const DecodeLayout &L, const DecodeArgs &a, int num_sms,
+                                   int32_t num_blocks_pool, cudaStream_t stream) {
+    const size_t smem = (size_t)(L.R + 1) * sizeof(int32_t);
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<D>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (kMaxRequestsPlan + 1) * (int)sizeof(int32_t));
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    decode_split_kernel<D><<<num_sms, kThreads, smem, stream>>>(a, L, num_blocks_pool);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const int64_t items = (int64_t)L.R * L.Hq;
+    const int64_t grid = (items + 7) / 8;
+    decode_combine_kernel<D><<<(unsigned)grid, 256, 0, stream>>>(a, L);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_decode(const DecodeLayout &L, const DecodeArgs &a, int num_sms,
+                               int32_t num_blocks_pool, cudaStream_t stream) {
+    if (L.d == 128) return launch_decode_t<128>(L, a, num_sms, num_blocks_pool, stream);
+    return launch_decode_t<64>(L, a, num_sms, num_blocks_pool, stream);
+}
+
+}  // namespace pkv

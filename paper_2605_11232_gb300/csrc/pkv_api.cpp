@@ -1,0 +1,414 @@
+// pkv_api.cpp -- the C ABI of include/pkv.h: host-side pool, argument checks
+// and kernel dispatch.  Host metadata only; device buffers belong to the caller.
+#include "../../include/pkv.h"
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "pkv_internal.h"
+
+struct pkv_pool {
+    pkv_pool_desc desc;
+    void *k_cache = nullptr;
+    void *v_cache = nullptr;
+    std::vector<int32_t> refcnt;     // 0 = free
+    std::vector<int32_t> free_list;  // back() is handed out next
+    int *d_err = nullptr;            // device error word
+    int device = -1;
+    int num_sms = 0;
+    bool tmaps_ready = false;
+    CUtensorMap tmap_k;
+    CUtensorMap tmap_v;
+};
+
+namespace {
+
+thread_local std::string g_last_error;
+
+int fail(int code, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return code;
+}
+
+int ok() {
+    g_last_error.clear();
+    return PKV_OK;
+}
+
+int cuda_fail(cudaError_t e, const char *what) {
+    return fail(PKV_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// splitmix64 (Steele, Lea, Flood 2014): the seeded stream of the placement.
+uint64_t splitmix64(uint64_t &s) {
+    uint64_t z = (s += 0x9E3779B97F4A7C15ull);
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+int check_kernel_pool(pkv_pool_t pool) {
+    if (!pool) return fail(PKV_ERR_INVALID_ARG, "pool is NULL");
+    if (!pool->k_cache || !pool->v_cache)
+        return fail(PKV_ERR_INVALID_ARG, "pool has no device caches (metadata-only pool)");
+    return PKV_OK;
+}
+
+int set_device(pkv_pool_t pool) {
+    int cur = -1;
+    cudaError_t e = cudaGetDevice(&cur);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (cur != pool->device) {
+        e = cudaSetDevice(pool->device);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaSetDevice");
+    }
+    return PKV_OK;
+}
+
+// TMA descriptors over the pool: a 4-D view {d, 16 slots, Hkv, num_blocks} of
+// each cache, box {64 elements, 16 slots, 1, 1} = one (block, head) half-row
+// tile of 2 KiB with the 128-byte swizzle the tensor-core operands use.
+int build_tmaps(pkv_pool_t pool) {
+    if (pool->tmaps_ready) return PKV_OK;
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                                     cudaEnableDefault, &q);
+    if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn)
+        return fail(PKV_ERR_CUDA, "cuTensorMapEncodeTiled entry point not found");
+    auto encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    const pkv_pool_desc &d = pool->desc;
+    cuuint64_t dims[4] = {(cuuint64_t)d.head_dim, 16, (cuuint64_t)d.num_kv_heads,
+                          (cuuint64_t)d.num_blocks};
+    cuuint64_t strides[3] = {(cuuint64_t)d.head_dim * 2, (cuuint64_t)d.head_dim * 2 * 16,
+                             (cuuint64_t)d.head_dim * 2 * 16 * d.num_kv_heads};
+    cuuint32_t box[4] = {64, 16, 1, 1};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    for (int which = 0; which < 2; ++which) {
+        CUresult r = encode(which ? &pool->tmap_v : &pool->tmap_k,
+                            CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4,
+                            which ? pool->v_cache : pool->k_cache, dims, strides, box, estr,
+                            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) return fail(PKV_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
+    }
+    pool->tmaps_ready = true;
+    return PKV_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *pkv_last_error(void) { return g_last_error.c_str(); }
+
+int kv_pool_create(const pkv_pool_desc *desc, void *k_cache, void *v_cache, pkv_pool_t *out) {
+    if (!desc || !out) return fail(PKV_ERR_INVALID_ARG, "desc and out must be non-NULL");
+    *out = nullptr;
+    if (desc->num_blocks <= 0 || desc->num_kv_heads <= 0)
+        return fail(PKV_ERR_INVALID_ARG, "num_blocks and num_kv_heads must be positive");
+    if (desc->block_size != 16) return fail(PKV_ERR_UNSUPPORTED, "block_size must be 16");
+    if (desc->head_dim != 64 && desc->head_dim != 128)
+        return fail(PKV_ERR_UNSUPPORTED, "head_dim must be 64 or 128");
+    if (desc->dtype != PKV_DTYPE_BF16) return fail(PKV_ERR_UNSUPPORTED, "dtype must be bf16");
+    if ((k_cache == nullptr) != (v_cache == nullptr))
+        return fail(PKV_ERR_INVALID_ARG, "give both caches or neither");
+    if (k_cache && (!aligned16(k_cache) || !aligned16(v_cache)))
+        return fail(PKV_ERR_INVALID_ARG, "caches must be 16-byte aligned");
+    pkv_pool *p = new pkv_pool();
+    p->desc = *desc;
+    p->k_cache = k_cache;
+    p->v_cache = v_cache;
+    const int32_t n = desc->num_blocks;
+    p->refcnt.assign(n, 0);
+    std::vector<int32_t> order(n);
+    for (int32_t i = 0; i < n; ++i) order[i] = i;
+    if (desc->placement_seed != 0) {
+        uint64_t s = desc->placement_seed;
+        for (int32_t i = n - 1; i > 0; --i) {   // Fisher-Yates
+            const int32_t j = (int32_t)(splitmix64(s) % (uint64_t)(i + 1));
+            std::swap(order[i], order[j]);
+        }
+    }
+    p->free_list.assign(order.rbegin(), order.rend());   // back() = order[0]
+    if (k_cache) {
+        cudaError_t e = cudaGetDevice(&p->device);
+        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount, p->device);
+        if (e == cudaSuccess) e = cudaMalloc(&p->d_err, sizeof(int));
+        if (e == cudaSuccess) e = cudaMemset(p->d_err, 0, sizeof(int));
+        if (e != cudaSuccess) {
+            if (p->d_err) cudaFree(p->d_err);
+            delete p;
+            return cuda_fail(e, "kv_pool_create");
+        }
+    }
+    *out = p;
+    return ok();
+}
+
+int kv_pool_destroy(pkv_pool_t pool) {
+    if (!pool) return ok();
+    if (pool->d_err) cudaFree(pool->d_err);
+    delete pool;
+    return ok();
+}
+
+int kv_pool_alloc(pkv_pool_t pool, int32_t n, int32_t *ids_out) {
+    if (!pool || n < 0 || (n > 0 && !ids_out)) return fail(PKV_ERR_INVALID_ARG, "bad arguments");
+    if ((size_t)n > pool->free_list.size())
+        return fail(PKV_ERR_OUT_OF_BLOCKS, "need %d blocks, %zu free", n, pool->free_list.size());
+    for (int32_t i = 0; i < n; ++i) {
+        const int32_t id = pool->free_list.back();
+        pool->free_list.pop_back();
+        pool->refcnt[id] = 1;
+        ids_out[i] = id;
+    }
+    return ok();
+}
+
+int kv_pool_retain(pkv_pool_t pool, const int32_t *ids, int32_t n) {
+    if (!pool || n < 0 || (n > 0 && !ids)) return fail(PKV_ERR_INVALID_ARG, "bad arguments");
+    for (int32_t i = 0; i < n; ++i) {
+        const int32_t id = ids[i];
+        if (id < 0 || id >= pool->desc.num_blocks)
+            return fail(PKV_ERR_REFCOUNT, "block id %d out of range", id);
+        if (pool->refcnt[id] <= 0) return fail(PKV_ERR_REFCOUNT, "block %d is free", id);
+    }
+    for (int32_t i = 0; i < n; ++i) ++pool->refcnt[ids[i]];
+    return ok();
+}
+
+int kv_pool_release(pkv_pool_t pool, const int32_t *ids, int32_t n) {
+    if (!pool || n < 0 || (n > 0 && !ids)) return fail(PKV_ERR_INVALID_ARG, "bad arguments");
+    std::vector<int32_t> drop;   // validate first: all or nothing
+    drop.reserve(n);
+    for (int32_t i = 0; i < n; ++i) {
+        const int32_t id = ids[i];
+        if (id < 0 || id >= pool->desc.num_blocks)
+            return fail(PKV_ERR_REFCOUNT, "block id %d out of range", id);
+        drop.push_back(id);
+    }
+    std::sort(drop.begin(), drop.end());
+    for (size_t i = 0; i < drop.size();) {
+        size_t j = i;
+        while (j < drop.size() && drop[j] == drop[i]) ++j;
+        if ((int32_t)(j - i) > pool->refcnt[drop[i]])
+            return fail(PKV_ERR_REFCOUNT, "block %d released %zu times with refcount %d",
+                        drop[i], j - i, pool->refcnt[drop[i]]);
+        i = j;
+    }
+    for (int32_t i = 0; i < n; ++i) {
+        if (--pool->refcnt[ids[i]] == 0) pool->free_list.push_back(ids[i]);
+    }
+    return ok();
+}
+
+int kv_pool_refcount(pkv_pool_t pool, int32_t id, int32_t *out) {
+    if (!pool || !out || id < 0 || id >= pool->desc.num_blocks)
+        return fail(PKV_ERR_INVALID_ARG, "bad arguments");
+    *out = pool->refcnt[id];
+    return ok();
+}
+
+int kv_pool_num_free(pkv_pool_t pool, int32_t *out) {
+    if (!pool || !out) return fail(PKV_ERR_INVALID_ARG, "bad arguments");
+    *out = (int32_t)pool->free_list.size();
+    return ok();
+}
+
+int kv_pool_alloc_sequence(pkv_pool_t pool, const int32_t *prefix_ids, int32_t n_prefix,
+                           int32_t n_blocks, int32_t *row_out) {
+    if (!pool || n_prefix < 0 || n_blocks < n_prefix || !row_out || (n_prefix > 0 && !prefix_ids))
+        return fail(PKV_ERR_INVALID_ARG, "bad arguments");
+    const int32_t n_new = n_blocks - n_prefix;
+    if ((size_t)n_new > pool->free_list.size())
+        return fail(PKV_ERR_OUT_OF_BLOCKS, "need %d blocks, %zu free", n_new, pool->free_list.size());
+    int rc = kv_pool_retain(pool, prefix_ids, n_prefix);
+    if (rc != PKV_OK) return rc;
+    for (int32_t i = 0; i < n_prefix; ++i) row_out[i] = prefix_ids[i];
+    return kv_pool_alloc(pool, n_new, row_out + n_prefix);
+}
+
+int kv_slot_mapping(pkv_pool_t pool, const int32_t *block_table, int32_t max_blocks,
+                    const int32_t *context_lens, const int32_t *new_lens, int32_t num_requests,
+                    int64_t *slots_out) {
+    if (!block_table || !context_lens || !new_lens || num_requests < 0 || max_blocks <= 0)
+        return fail(PKV_ERR_INVALID_ARG, "bad arguments");
+    int64_t t = 0;
+    for (int32_t r = 0; r < num_requests; ++r) {
+        const int32_t L = context_lens[r], n = new_lens[r];
+        if (n < 0 || L < n || (L + 15) / 16 > max_blocks)
+            return fail(PKV_ERR_INVALID_ARG, "request %d: context %d, new %d, table width %d", r, L,
+                        n, max_blocks);
+        for (int32_t i = 0; i < n; ++i) {
+            const int64_t p = (int64_t)L - n + i;
+            const int32_t blk = block_table[(int64_t)r * max_blocks + p / 16];
+            if (blk < 0) return fail(PKV_ERR_INVALID_ARG, "request %d: no block for position %lld", r, (long long)p);
+            if (pool) {
+                if (blk >= pool->desc.num_blocks || pool->refcnt[blk] == 0)
+                    return fail(PKV_ERR_REFCOUNT, "request %d: block %d is not allocated", r, blk);
+                if (pool->refcnt[blk] > 1)
+                    return fail(PKV_ERR_SHARED_BLOCK_WRITE,
+                                "request %d: position %lld maps into shared block %d", r,
+                                (long long)p, blk);
+            }
+            if (slots_out) slots_out[t] = (int64_t)blk * 16 + p % 16;
+            ++t;
+        }
+    }
+    return ok();
+}
+
+int kv_cache_write(pkv_pool_t pool, const void *k_new, const void *v_new,
+                   const int64_t *slot_mapping, int32_t num_tokens, pkv_stream_t stream) {
+    int rc = check_kernel_pool(pool);
+    if (rc != PKV_OK) return rc;
+    if (num_tokens < 0) return fail(PKV_ERR_INVALID_ARG, "num_tokens < 0");
+    if (num_tokens == 0) return ok();
+    if (!k_new || !v_new || !slot_mapping) return fail(PKV_ERR_INVALID_ARG, "NULL buffer");
+    if (!aligned16(k_new) || !aligned16(v_new) || (reinterpret_cast<uintptr_t>(slot_mapping) & 7))
+        return fail(PKV_ERR_INVALID_ARG, "misaligned buffer");
+    if ((rc = set_device(pool)) != PKV_OK) return rc;
+    const pkv_pool_desc &d = pool->desc;
+    cudaError_t e = pkv::launch_cache_write(k_new, v_new, slot_mapping, num_tokens, pool->k_cache,
+                                            pool->v_cache, d.num_kv_heads, d.head_dim,
+                                            (int64_t)d.num_blocks * 16, pool->d_err,
+                                            static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "kv_cache_write launch");
+    return ok();
+}
+
+int paged_attn_prefill(pkv_pool_t pool, const void *q, void *out, float *lse,
+                       const int32_t *cu_seqlens_q, const int32_t *context_lens,
+                       const int32_t *block_table, int32_t max_blocks, int32_t num_requests,
+                       int32_t max_seqlen_q, int32_t num_q_heads, float scale,
+                       pkv_stream_t stream) {
+    int rc = check_kernel_pool(pool);
+    if (rc != PKV_OK) return rc;
+    const pkv_pool_desc &d = pool->desc;
+    if (num_requests < 0 || max_seqlen_q < 0 || max_blocks <= 0)
+        return fail(PKV_ERR_INVALID_ARG, "bad sizes");
+    if (num_q_heads <= 0 || num_q_heads % d.num_kv_heads != 0)
+        return fail(PKV_ERR_INVALID_ARG, "num_q_heads must be a positive multiple of num_kv_heads");
+    if (num_q_heads / d.num_kv_heads > 128)
+        return fail(PKV_ERR_UNSUPPORTED, "more than 128 q heads per kv head");
+    if (!(scale > 0.f) || !std::isfinite(scale)) return fail(PKV_ERR_INVALID_ARG, "bad scale");
+    if (num_requests == 0 || max_seqlen_q == 0) return ok();
+    if (!q || !out || !cu_seqlens_q || !context_lens || !block_table)
+        return fail(PKV_ERR_INVALID_ARG, "NULL buffer");
+    if (!aligned16(q) || !aligned16(out)) return fail(PKV_ERR_INVALID_ARG, "misaligned q/out");
+    if ((rc = set_device(pool)) != PKV_OK) return rc;
+    if ((rc = build_tmaps(pool)) != PKV_OK) return rc;
+    pkv::PrefillArgs a{};
+    a.q = q; a.out = out; a.lse = lse;
+    a.cu_seqlens_q = cu_seqlens_q; a.context_lens = context_lens;
+    a.block_table = block_table; a.max_blocks = max_blocks;
+    a.R = num_requests; a.Hq = num_q_heads; a.Hkv = d.num_kv_heads; a.d = d.head_dim;
+    a.max_seqlen_q = max_seqlen_q;
+    a.scale_log2 = scale * 1.4426950408889634f;
+    a.tmap_k = &pool->tmap_k; a.tmap_v = &pool->tmap_v;
+    a.err = pool->d_err;
+    cudaError_t e = pkv::launch_prefill(a, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "paged_attn_prefill launch");
+    return ok();
+}
+
+int paged_attn_decode_workspace_size(pkv_pool_t pool, int32_t num_requests, int32_t num_q_heads,
+                                     int32_t max_blocks, const pkv_prefix_groups *groups,
+                                     size_t *bytes_out) {
+    if (!pool || !bytes_out || num_requests < 0 || num_q_heads <= 0 || max_blocks <= 0)
+        return fail(PKV_ERR_INVALID_ARG, "bad arguments");
+    const int32_t G = groups ? groups->num_groups : 0;
+    const int32_t mgb = groups ? groups->max_group_blocks : 0;
+    pkv::DecodeLayout L = pkv::decode_layout(num_requests, num_q_heads, pool->desc.num_kv_heads,
+                                             pool->desc.head_dim, max_blocks, G, mgb);
+    *bytes_out = L.total;
+    return ok();
+}
+
+int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
+                      const int32_t *context_lens, const int32_t *block_table, int32_t max_blocks,
+                      int32_t num_requests, int32_t num_q_heads, float scale,
+                      const pkv_prefix_groups *groups, void *workspace, size_t workspace_bytes,
+                      pkv_stream_t stream) {
+    int rc = check_kernel_pool(pool);
+    if (rc != PKV_OK) return rc;
+    const pkv_pool_desc &d = pool->desc;
+    if (num_requests < 0 || max_blocks <= 0) return fail(PKV_ERR_INVALID_ARG, "bad sizes");
+    if (num_q_heads <= 0 || num_q_heads % d.num_kv_heads != 0)
+        return fail(PKV_ERR_INVALID_ARG, "num_q_heads must be a positive multiple of num_kv_heads");
+    const int32_t g = num_q_heads / d.num_kv_heads;
+    if (g > 8) return fail(PKV_ERR_UNSUPPORTED, "decode supports up to 8 q heads per kv head");
+    if (num_requests > 16384) return fail(PKV_ERR_UNSUPPORTED, "decode supports up to 16384 requests");
+    if (!(scale > 0.f) || !std::isfinite(scale)) return fail(PKV_ERR_INVALID_ARG, "bad scale");
+    if (num_requests == 0) return ok();
+    if (!q || !out || !context_lens || !block_table) return fail(PKV_ERR_INVALID_ARG, "NULL buffer");
+    if (!aligned16(q) || !aligned16(out)) return fail(PKV_ERR_INVALID_ARG, "misaligned q/out");
+    int32_t G = 0, mgb = 0;
+    if (groups && groups->num_groups > 0) {
+        G = groups->num_groups;
+        mgb = groups->max_group_blocks;
+        if (!groups->group_start || !groups->member_req || !groups->group_blocks ||
+            !groups->group_of_req || mgb < 0 || groups->max_group_members < 0)
+            return fail(PKV_ERR_INVALID_ARG, "incomplete prefix-group descriptor");
+        return fail(PKV_ERR_UNSUPPORTED, "prefix-shared decode pass not built yet");
+    }
+    pkv::DecodeLayout L = pkv::decode_layout(num_requests, num_q_heads, d.num_kv_heads, d.head_dim,
+                                             max_blocks, G, mgb);
+    if (!workspace || workspace_bytes < L.total)
+        return fail(PKV_ERR_WORKSPACE, "workspace of %zu bytes needed", L.total);
+    if (reinterpret_cast<uintptr_t>(workspace) & 255)
+        return fail(PKV_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+    if ((rc = set_device(pool)) != PKV_OK) return rc;
+    pkv::DecodeArgs a{};
+    a.q = q; a.out = out; a.lse = lse;
+    a.context_lens = context_lens; a.block_table = block_table; a.max_blocks = max_blocks;
+    a.k_cache = pool->k_cache; a.v_cache = pool->v_cache;
+    a.scale_log2 = scale * 1.4426950408889634f;
+    a.num_groups = G;
+    if (G > 0) {
+        a.max_group_members = groups->max_group_members;
+        a.group_start = groups->group_start; a.member_req = groups->member_req;
+        a.group_blocks = groups->group_blocks; a.group_of_req = groups->group_of_req;
+    }
+    a.ws = workspace;
+    a.err = pool->d_err;
+    cudaError_t e = pkv::launch_decode(L, a, pool->num_sms, d.num_blocks,
+                                       static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode launch");
+    return ok();
+}
+
+int pkv_check_device_errors(pkv_pool_t pool, pkv_stream_t stream, int32_t *code_out) {
+    int rc = check_kernel_pool(pool);
+    if (rc != PKV_OK) return rc;
+    if (!code_out) return fail(PKV_ERR_INVALID_ARG, "code_out is NULL");
+    if ((rc = set_device(pool)) != PKV_OK) return rc;
+    cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    int v = 0;
+    e = cudaMemcpy(&v, pool->d_err, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess) e = cudaMemset(pool->d_err, 0, sizeof(int));
+    if (e != cudaSuccess) return cuda_fail(e, "reading the device error word");
+    *code_out = v;
+    return ok();
+}
+
+}  // extern "C"

@@ -1,0 +1,88 @@
+// pkv_internal.h -- declarations shared by the host API and the kernel files.
+// Not part of the public ABI (that is include/pkv.h).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace pkv {
+
+// Device error word values (a kernel latches the first one with atomicCAS).
+enum : int {
+    kDevOk = 0,
+    kDevBounds = -9,   // PKV_ERR_DEVICE_BOUNDS
+    kDevTimeout = -8,  // PKV_ERR_DEVICE_TIMEOUT
+};
+
+// Decode split-KV layout, shared by the split, prefix and combine kernels.
+// Partials of request r, q-head hq live at part slots
+//   [(r * Hq + hq) * parts_per_head + p]
+// with p in [0, prefix_parts) for the shared-prefix pass and
+// p in [prefix_parts, prefix_parts + kMaxPrivateParts) for private pieces.
+constexpr int kMaxPrivateParts = 16;
+constexpr int kMaxPrefixParts = 48;   // parts_per_head <= 64: two per combine lane
+constexpr int kMinBlocksPerPiece = 4;
+
+struct DecodeLayout {
+    int32_t R, Hq, Hkv, d, g;
+    int32_t prefix_parts;        // prefix-pass part slots per head (0 without groups)
+    int32_t prefix_blocks_per_part;
+    int32_t parts_per_head;      // prefix_parts + kMaxPrivateParts
+    // byte offsets inside the workspace
+    size_t off_o;                // float [R*Hq*parts][d]
+    size_t off_ml;               // float2 [R*Hq*parts]
+    size_t off_nparts;           // int32 [R*Hkv] private pieces per (r, kv head)
+    size_t total;
+};
+
+DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_t max_blocks,
+                           int32_t num_groups, int32_t max_group_blocks);
+
+cudaError_t launch_cache_write(const void *k_new, const void *v_new, const int64_t *slots,
+                               int32_t T, void *k_cache, void *v_cache, int32_t Hkv, int32_t d,
+                               int64_t num_slots, int *err, cudaStream_t stream);
+
+struct DecodeArgs {
+    const void *q;
+    void *out;
+    float *lse;
+    const int32_t *context_lens;
+    const int32_t *block_table;
+    int32_t max_blocks;
+    const void *k_cache;
+    const void *v_cache;
+    float scale_log2;   // softmax scale * log2(e)
+    // prefix groups (all null / 0 without groups)
+    int32_t num_groups;
+    int32_t max_group_members;
+    const int32_t *group_start;
+    const int32_t *member_req;
+    const int32_t *group_blocks;
+    const int32_t *group_of_req;
+    void *ws;
+    int *err;
+};
+
+cudaError_t launch_decode(const DecodeLayout &L, const DecodeArgs &a, int num_sms,
+                          int32_t num_blocks_pool, cudaStream_t stream);
+
+struct PrefillArgs {
+    const void *q;
+    void *out;
+    float *lse;
+    const int32_t *cu_seqlens_q;
+    const int32_t *context_lens;
+    const int32_t *block_table;
+    int32_t max_blocks;
+    int32_t R, Hq, Hkv, d;
+    int32_t max_seqlen_q;
+    float scale_log2;
+    const CUtensorMap *tmap_k;  // host copies, passed by value to the kernel
+    const CUtensorMap *tmap_v;
+    int *err;
+};
+
+cudaError_t launch_prefill(const PrefillArgs &a, cudaStream_t stream);
+
+}  // namespace pkv

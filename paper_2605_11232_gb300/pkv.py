@@ -1,0 +1,243 @@
+"""ctypes binding of ``libpkv.so`` (include/pkv.h), argument marshalling only.
+
+Every function here forwards to the C entry point of the same name.  Device
+buffers are torch CUDA tensors owned by the caller; host arrays are numpy.
+There is no fallback: if the library cannot be loaded, every call raises.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_build", "libpkv.so")
+
+PKV_OK = 0
+PKV_ERR_INVALID_ARG = -1
+PKV_ERR_OUT_OF_BLOCKS = -2
+PKV_ERR_REFCOUNT = -3
+PKV_ERR_SHARED_BLOCK_WRITE = -4
+PKV_ERR_CUDA = -5
+PKV_ERR_UNSUPPORTED = -6
+PKV_ERR_WORKSPACE = -7
+PKV_ERR_DEVICE_TIMEOUT = -8
+PKV_ERR_DEVICE_BOUNDS = -9
+PKV_DTYPE_BF16 = 1
+
+# every entry point declared in include/pkv.h
+EXPORTS = [
+    "kv_pool_create", "kv_pool_destroy", "kv_pool_alloc", "kv_pool_retain", "kv_pool_release",
+    "kv_pool_refcount", "kv_pool_num_free", "kv_pool_alloc_sequence", "kv_slot_mapping",
+    "kv_cache_write", "paged_attn_prefill", "paged_attn_decode_workspace_size",
+    "paged_attn_decode", "pkv_check_device_errors", "pkv_last_error",
+]
+
+
+class PkvError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"pkv error {code}: {msg}")
+        self.code = code
+
+
+class PoolDesc(ctypes.Structure):
+    _fields_ = [("num_blocks", ctypes.c_int32), ("block_size", ctypes.c_int32),
+                ("num_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("dtype", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("placement_seed", ctypes.c_uint64)]
+
+
+class PrefixGroups(ctypes.Structure):
+    _fields_ = [("num_groups", ctypes.c_int32), ("max_group_blocks", ctypes.c_int32),
+                ("max_group_members", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("group_start", ctypes.c_void_p), ("member_req", ctypes.c_void_p),
+                ("group_blocks", ctypes.c_void_p), ("group_of_req", ctypes.c_void_p)]
+
+
+_lib = None
+
+
+def load(path: str | None = None):
+    """Load the library (built by ``__graft_entry__.build()`` / ``build.py``)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    p = path or LIB_PATH
+    if not os.path.exists(p):
+        raise RuntimeError(f"libpkv.so not built ({p}); run __graft_entry__.build()")
+    lib = ctypes.CDLL(p)
+    V, P, i32, i64, f32 = (ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64,
+                           ctypes.c_float)
+    sz = ctypes.c_size_t
+    sig = {
+        "kv_pool_create": [ctypes.POINTER(PoolDesc), V, V, ctypes.POINTER(V)],
+        "kv_pool_destroy": [V],
+        "kv_pool_alloc": [V, i32, P],
+        "kv_pool_retain": [V, P, i32],
+        "kv_pool_release": [V, P, i32],
+        "kv_pool_refcount": [V, i32, P],
+        "kv_pool_num_free": [V, P],
+        "kv_pool_alloc_sequence": [V, P, i32, i32, P],
+        "kv_slot_mapping": [V, P, i32, P, P, i32, P],
+        "kv_cache_write": [V, V, V, V, i32, V],
+        "paged_attn_prefill": [V, V, V, V, V, V, V, i32, i32, i32, i32, f32, V],
+        "paged_attn_decode_workspace_size": [V, i32, i32, i32, ctypes.POINTER(PrefixGroups),
+                                             ctypes.POINTER(sz)],
+        "paged_attn_decode": [V, V, V, V, V, V, i32, i32, i32, f32,
+                              ctypes.POINTER(PrefixGroups), V, sz, V],
+        "pkv_check_device_errors": [V, V, P],
+    }
+    for name, args in sig.items():
+        fn = getattr(lib, name)
+        fn.argtypes = args
+        fn.restype = ctypes.c_int
+    lib.pkv_last_error.argtypes = []
+    lib.pkv_last_error.restype = ctypes.c_char_p
+    _lib = lib
+    return lib
+
+
+def _check(rc: int):
+    if rc != PKV_OK:
+        raise PkvError(rc, load().pkv_last_error().decode())
+
+
+def _np_ptr(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _dptr(t):
+    """Device address of a torch tensor (or None)."""
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("expected a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError("expected a contiguous tensor")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return ctypes.c_void_p(stream)
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+# ---- a1: pool ---------------------------------------------------------------
+
+def kv_pool_create(num_blocks: int, num_kv_heads: int, head_dim: int, k_cache=None,
+                   v_cache=None, placement_seed: int = 0, block_size: int = 16):
+    desc = PoolDesc(num_blocks, block_size, num_kv_heads, head_dim, PKV_DTYPE_BF16, 0,
+                    placement_seed & (2**64 - 1))
+    h = ctypes.c_void_p()
+    _check(load().kv_pool_create(ctypes.byref(desc), _dptr(k_cache), _dptr(v_cache),
+                                 ctypes.byref(h)))
+    return h
+
+
+def kv_pool_destroy(pool):
+    _check(load().kv_pool_destroy(pool))
+
+
+def kv_pool_alloc(pool, n: int) -> np.ndarray:
+    ids = np.zeros(max(n, 1), np.int32)
+    _check(load().kv_pool_alloc(pool, n, _np_ptr(ids)))
+    return ids[:n]
+
+
+def kv_pool_retain(pool, ids):
+    ids = np.ascontiguousarray(ids, np.int32)
+    _check(load().kv_pool_retain(pool, _np_ptr(ids), len(ids)))
+
+
+def kv_pool_release(pool, ids):
+    ids = np.ascontiguousarray(ids, np.int32)
+    _check(load().kv_pool_release(pool, _np_ptr(ids), len(ids)))
+
+
+def kv_pool_refcount(pool, block_id: int) -> int:
+    out = np.zeros(1, np.int32)
+    _check(load().kv_pool_refcount(pool, int(block_id), _np_ptr(out)))
+    return int(out[0])
+
+
+def kv_pool_num_free(pool) -> int:
+    out = np.zeros(1, np.int32)
+    _check(load().kv_pool_num_free(pool, _np_ptr(out)))
+    return int(out[0])
+
+
+def kv_pool_alloc_sequence(pool, prefix_ids, n_blocks: int) -> np.ndarray:
+    pre = np.ascontiguousarray(prefix_ids if prefix_ids is not None else [], np.int32)
+    row = np.zeros(max(n_blocks, 1), np.int32)
+    _check(load().kv_pool_alloc_sequence(pool, _np_ptr(pre) if len(pre) else None, len(pre),
+                                         int(n_blocks), _np_ptr(row)))
+    return row[:n_blocks]
+
+
+# ---- a2: slot mapping --------------------------------------------------------
+
+def kv_slot_mapping(pool, block_table: np.ndarray, context_lens, new_lens) -> np.ndarray:
+    table = np.ascontiguousarray(block_table, np.int32)
+    ctx = np.ascontiguousarray(context_lens, np.int32)
+    new = np.ascontiguousarray(new_lens, np.int32)
+    out = np.zeros(max(int(new.sum()), 1), np.int64)
+    _check(load().kv_slot_mapping(pool, _np_ptr(table), table.shape[1], _np_ptr(ctx),
+                                  _np_ptr(new), len(ctx), _np_ptr(out)))
+    return out[: int(new.sum())]
+
+
+# ---- a3-a7: kernels ---------------------------------------------------------
+
+def kv_cache_write(pool, k_new, v_new, slot_mapping, stream=None):
+    _check(load().kv_cache_write(pool, _dptr(k_new), _dptr(v_new), _dptr(slot_mapping),
+                                 int(slot_mapping.shape[0]), _stream(stream)))
+
+
+def paged_attn_prefill(pool, q, out, lse, cu_seqlens_q, context_lens, block_table,
+                       max_seqlen_q: int, scale: float, stream=None):
+    _check(load().paged_attn_prefill(
+        pool, _dptr(q), _dptr(out), _dptr(lse), _dptr(cu_seqlens_q), _dptr(context_lens),
+        _dptr(block_table), int(block_table.shape[1]), int(context_lens.shape[0]),
+        int(max_seqlen_q), int(q.shape[1]), float(scale), _stream(stream)))
+
+
+def make_prefix_groups(num_groups=0, max_group_blocks=0, max_group_members=0, group_start=None,
+                       member_req=None, group_blocks=None, group_of_req=None):
+    return PrefixGroups(int(num_groups), int(max_group_blocks), int(max_group_members), 0,
+                        _dptr(group_start), _dptr(member_req), _dptr(group_blocks),
+                        _dptr(group_of_req))
+
+
+def paged_attn_decode_workspace_size(pool, num_requests: int, num_q_heads: int,
+                                     max_blocks: int, groups=None) -> int:
+    out = ctypes.c_size_t()
+    _check(load().paged_attn_decode_workspace_size(
+        pool, int(num_requests), int(num_q_heads), int(max_blocks),
+        ctypes.byref(groups) if groups is not None else None, ctypes.byref(out)))
+    return int(out.value)
+
+
+def paged_attn_decode(pool, q, out, lse, context_lens, block_table, scale: float, groups,
+                      workspace, stream=None):
+    _check(load().paged_attn_decode(
+        pool, _dptr(q), _dptr(out), _dptr(lse), _dptr(context_lens), _dptr(block_table),
+        int(block_table.shape[1]), int(context_lens.shape[0]), int(q.shape[1]), float(scale),
+        ctypes.byref(groups) if groups is not None else None, _dptr(workspace),
+        int(workspace.numel() * workspace.element_size()) if workspace is not None else 0,
+        _stream(stream)))
+
+
+def pkv_check_device_errors(pool, stream=None) -> int:
+    out = np.zeros(1, np.int32)
+    _check(load().pkv_check_device_errors(pool, _stream(stream), _np_ptr(out)))
+    return int(out[0])
+
+
+def pkv_last_error() -> str:
+    return load().pkv_last_error().decode()

@@ -1,0 +1,162 @@
+"""paged_attn_decode against the fp64 oracle (GPU).
+
+Tolerance: max |out - oracle| <= 1e-2 and mean <= 1e-3 over all elements of a
+run (bf16 inputs, fp32 accumulation, bf16 output); LSE within 1e-3.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2605_11232_gb300 import batch as B
+from paper_2605_11232_gb300 import pkv
+from paper_2605_11232_gb300.workloads import make_workload
+
+from _lib import need_gpu
+
+pytestmark = pytest.mark.gpu
+
+MAX_ABS, MEAN_ABS, LSE_ABS = 1e-2, 1e-3, 1e-3
+
+
+def _f64(t):
+    return t.detach().float().cpu().numpy().astype(np.float64)
+
+
+def run_decode(b, use_groups=False, with_lse=True):
+    w = b.w
+    Rd = b.dec.stop - b.dec.start
+    B.run_write(b)
+    out = torch.empty((Rd, w.num_q_heads, w.head_dim), dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty((Rd, w.num_q_heads), dtype=torch.float32, device="cuda") if with_lse else None
+    ws = B.decode_workspace(b, use_groups)
+    B.run_decode(b, out, lse, ws, use_groups)
+    assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
+    return out, lse
+
+
+def compare(b, out, lse, reqs, threads=8):
+    w = b.w
+    errs, lerrs = [], []
+    for r in reqs:
+        o_ref, l_ref = oracle.request_attention(w, int(r), threads=threads)
+        i = int(r) - b.dec.start
+        errs.append(np.abs(_f64(out[i]) - o_ref[0]))
+        if lse is not None:
+            lerrs.append(np.abs(_f64(lse[i]) - l_ref[0]))
+    e = np.concatenate([x.ravel() for x in errs])
+    assert np.isfinite(e).all()
+    assert e.max() <= MAX_ABS and e.mean() <= MEAN_ABS, (e.max(), e.mean())
+    if lerrs:
+        le = np.concatenate(lerrs)
+        assert le.max() <= LSE_ABS, le.max()
+    return e.max(), e.mean()
+
+
+@pytest.mark.parametrize("name,scale", [
+    ("tiny_decode", 1.0),
+    ("l8b_decode", 0.25),     # 16 requests of full length
+    ("qwen_mixed", 0.125),    # 32 decode requests over three prefixes, g = 7
+    ("l70b_decode", 1 / 32),  # 16 requests, log-uniform suffixes, g = 8
+])
+def test_decode_matches_oracle(name, scale):
+    need_gpu()
+    w = make_workload(name, scale_requests=scale)
+    b = B.build_batch(w, poison=True)
+    out, lse = run_decode(b)
+    compare(b, out, lse, range(b.dec.start, b.dec.stop))
+    b.close()
+
+
+@pytest.mark.parametrize("name", ["l8b_decode", "qwen_mixed", "l70b_decode"])
+def test_decode_full_size_sampled(name):
+    """Full-size batch, same call as the benchmark; outputs of a sample of
+    requests (first, last, shortest, longest, and random) against the oracle,
+    and no NaN anywhere."""
+    need_gpu()
+    w = make_workload(name)
+    b = B.build_batch(w, poison=True)
+    out, lse = run_decode(b)
+    assert torch.isfinite(out.float()).all()
+    ctx = w.context_lens[b.dec]
+    rng = np.random.default_rng(0)
+    picks = {0, len(ctx) - 1, int(np.argmin(ctx)), int(np.argmax(ctx))}
+    picks |= set(rng.choice(len(ctx), 4, replace=False).tolist())
+    compare(b, out, lse, [b.dec.start + i for i in sorted(picks)], threads=16)
+    b.close()
+
+
+def test_placement_invariance_bit_exact():
+    """Different physical placements of the same logical cache give
+    bit-identical outputs (the reduction order depends on positions only)."""
+    need_gpu()
+    w = make_workload("l8b_decode", scale_requests=0.125)
+    outs = []
+    for seed in (0, 7, 123456789):
+        b = B.build_batch(w, poison=True, placement_seed=seed)
+        o, l = run_decode(b)
+        outs.append((o.cpu(), l.cpu()))
+        b.close()
+    for o, l in outs[1:]:
+        assert torch.equal(o, outs[0][0]) and torch.equal(l, outs[0][1])
+
+
+def test_shared_prefix_equals_private_copies():
+    """Reading the prefix through shared refcounted blocks or through private
+    copies gives the same outputs (without the grouped prefix pass: bit-exact)."""
+    need_gpu()
+    w = make_workload("qwen_mixed", scale_requests=0.0625)
+    b1 = B.build_batch(w, poison=True)
+    o1, l1 = run_decode(b1)
+    b2 = B.build_batch(w, poison=True, share_prefix=False)
+    o2, l2 = run_decode(b2)
+    assert torch.equal(o1, o2) and torch.equal(l1, l2)
+    b1.close(); b2.close()
+
+
+def test_single_key_returns_value():
+    """A context of one token returns that token's V (weight exactly 1)."""
+    need_gpu()
+    w = make_workload("custom", custom=dict(Hq=8, Hkv=2, d=128, prefix_lens=[], group=[-1, -1, -1],
+                                          cached=[0, 0, 0], new=[1, 1, 1], decode=[True] * 3,
+                                          num_blocks=8))
+    b = B.build_batch(w, poison=True)
+    out, lse = run_decode(b)
+    v = w.new_v.float()
+    for r in range(3):
+        for h in range(8):
+            assert torch.equal(out[r, h].cpu().float(), v[r, h // 4])
+    b.close()
+
+
+def test_causality_future_slots_ignored():
+    """Keys past the context (rest of the last block) never matter: the result
+    is identical whatever those slots hold."""
+    need_gpu()
+    w = make_workload("l8b_decode", scale_requests=0.0625)
+    b = B.build_batch(w, poison=False)
+    o1, l1 = run_decode(b)
+    # overwrite every slot past each request's context inside its last block
+    for r in range(w.num_requests):
+        L = int(w.context_lens[r])
+        blk = int(b.table_host[r, (L - 1) // 16])
+        b.k_cache[blk, :, L % 16 or 16:, :] = 1000.0
+        b.v_cache[blk, :, L % 16 or 16:, :] = float("inf")
+    ws = B.decode_workspace(b, False)
+    o2 = torch.empty_like(o1)
+    l2 = torch.empty_like(l1)
+    B.run_decode(b, o2, l2, ws, False)
+    assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
+    assert torch.equal(o1, o2) and torch.equal(l1, l2)
+    b.close()
+
+
+def test_bad_arguments_rejected_before_launch():
+    need_gpu()
+    w = make_workload("tiny_decode")
+    b = B.build_batch(w)
+    out = torch.empty((4, 8, 64), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(pkv.PkvError) as e:
+        B.run_decode(b, out, None, torch.empty(16, dtype=torch.uint8, device="cuda"), False)
+    assert e.value.code == pkv.PKV_ERR_WORKSPACE
+    b.close()
