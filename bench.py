@@ -1,0 +1,497 @@
+#!/usr/bin/env python
+"""Benchmark of the prefix-cached paged-attention path on GB300.
+
+One step = one pass of the hot path over one batch: the new tokens' K/V are
+scattered into the paged pool (kv_cache_write), then the batch's attention runs
+(paged_attn_decode for decode requests, paged_attn_prefill for suffix or chunk
+prefills).  The headline workload is the Llama-3-8B-shaped decode batch
+(64 requests sharing a 4096-token policy prefix); its metric is HBM GB/s on
+algorithmic bytes (every distinct K/V row read once, shared prefix rows once,
+plus the step's Q, O and new-token K/V traffic).  Other workloads are reported
+under "workloads" (prefill in TFLOP/s on visible query-key pairs).
+
+Timing: per-step CUDA events on the launching stream, L2 flushed (256 MiB
+write) before every step outside the events, W warm-up steps, max over ranks.
+Per-kernel times come from the library's own event tracing (pkv_trace_*).
+
+--impl reference times the fp64 CPU oracle (the only reference this path has)
+on the host cores, one decode request per step.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+HEADLINE = "l8b_decode"
+WORKLOAD_DESC = {
+    "tiny": "tiny: 8q/2kv heads, d64, 4 requests sharing a 256-token prefix, suffix prefill",
+    "l8b_decode": "l8b_decode: Llama-3-8B-shaped decode, 32q/8kv heads, d128, 64 requests "
+                  "sharing a 4096-token prefix, suffix U[256,1024], generated U[0,128]",
+    "l8b_prefill": "l8b_prefill: Llama-3-8B-shaped suffix prefill, 32q/8kv, d128, 32 requests, "
+                   "cached 4096-token prefix, suffix U[512,1024]",
+    "qwen_mixed": "qwen_mixed: Qwen2.5-7B-shaped, 28q/4kv, d128, 256 decode requests over "
+                  "2048/4096/6144-token prefixes + 8 chunked prefills of 512",
+    "l70b_decode": "l70b_decode: Llama-3-70B-shaped decode, 64q/8kv, d128, 512 requests sharing "
+                   "a 6144-token prefix, suffix log-U[64,2048], generated U[0,128]",
+}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), float(d["bf16_tflops_sustained"]), "measured"
+    return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# algorithmic work (counted from the workload's lengths, not from the kernels)
+
+def kv_row_bytes(w):
+    return 2 * w.num_kv_heads * w.head_dim * 2      # K and V of one token, all kv heads
+
+
+def decode_bytes(w, req):
+    """Distinct K/V rows of the decode requests (shared prefix once) + Q + O."""
+    rows = 0
+    groups = set()
+    for r in range(req.start, req.stop):
+        g = int(w.group_of_req[r])
+        if g >= 0:
+            groups.add(g)
+        rows += int(w.context_lens[r]) - w.prefix_len_of(r)
+    rows += sum(w.prefix_lens[g] for g in groups)
+    nq = req.stop - req.start
+    return rows * kv_row_bytes(w) + 2 * nq * w.num_q_heads * w.head_dim * 2
+
+
+def write_bytes(w, ntok):
+    return 2 * ntok * kv_row_bytes(w)                # read new K/V + write into the pool
+
+
+def prefill_flops(w, req):
+    """4 * d * Hq * visible (query, key) pairs; masked pairs are not counted."""
+    pairs = 0
+    for r in range(req.start, req.stop):
+        S, c = int(w.new_lens[r]), int(w.cached_lens[r])
+        pairs += S * c + S * (S + 1) // 2
+    return 4 * w.head_dim * w.num_q_heads * pairs
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.samples = []   # (t, sm, smmax, reasons)
+        self.proc = None
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm, smmax = float(parts[1]), float(parts[2])
+            except ValueError:
+                continue
+            reasons = [n for n, v in zip(names, parts[5:9]) if v.lower().startswith("active")]
+            self.samples.append((time.time(), sm, smmax, reasons))
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self, t0, t1):
+        inside = [s for s in self.samples if t0 <= s[0] <= t1]
+        use = inside if inside else self.samples
+        if not use:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        reasons = sorted({r for s in use for r in s[3]})
+        return {"sm_mhz": statistics.median(s[1] for s in use), "sm_max_mhz": max(s[2] for s in use),
+                "reasons": reasons, "samples": len(use),
+                "window": "timed region" if inside else "whole run (timed region shorter than the 100 ms sampling)"}
+
+
+# ---------------------------------------------------------------------------
+
+def dist_setup(n_gpus):
+    import torch
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x, world):
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(x, world):
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+def ncu_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary, if the
+    kernel source is unchanged since the capture."""
+    p = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    if not os.path.exists(p):
+        return None
+    d = json.load(open(p)).get(kernel)
+    if not d or d.get("workload") != workload:
+        return None
+    src = os.path.join(ROOT, d["source"])
+    if not os.path.exists(src) or hashlib.sha256(open(src, "rb").read()).hexdigest() != d["source_sha256"]:
+        return None
+    return d["dram_bytes_per_launch"]
+
+
+def run_steps(step_fn, flush, steps, stream):
+    """Per-step CUDA events around step_fn on `stream`, L2 flush before each
+    step (outside the events)."""
+    import torch
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(steps)]
+    for a, b in evs:
+        flush()
+        a.record(stream)
+        step_fn()
+        b.record(stream)
+    torch.cuda.synchronize()
+    return [a.elapsed_time(b) for a, b in evs]
+
+
+def measure_workload(name, steps, warmup, use_groups=True, e2e_steps=0):
+    """Build a workload, time its steps; returns a dict of results."""
+    import numpy as np
+    import torch
+
+    from paper_2605_11232_gb300 import batch as B
+    from paper_2605_11232_gb300 import pkv
+    from paper_2605_11232_gb300.workloads import make_workload
+
+    w = make_workload(name)
+    b = B.build_batch(w, poison=False)
+    stream = torch.cuda.current_stream()
+    dev = b.device
+    Rd, Rp = b.dec.stop - b.dec.start, b.pre.stop - b.pre.start
+    out_d = torch.empty((Rd, w.num_q_heads, w.head_dim), dtype=torch.bfloat16, device=dev)
+    rows_p = B.new_token_rows(w, b.pre)
+    out_p = torch.empty((rows_p.stop - rows_p.start, w.num_q_heads, w.head_dim),
+                        dtype=torch.bfloat16, device=dev)
+    groups_ok = use_groups and b.groups is not None
+    ws = B.decode_workspace(b, groups_ok) if Rd else None
+    flush_buf = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)
+
+    def flush():
+        flush_buf.fill_(1)
+
+    def step():
+        B.run_write(b)
+        if Rp:
+            B.run_prefill(b, out_p, None)
+        if Rd:
+            B.run_decode(b, out_d, None, ws, groups_ok)
+
+    # check the configuration runs (prefix pass may be unavailable)
+    try:
+        step()
+    except pkv.PkvError as e:
+        if groups_ok and e.code == pkv.PKV_ERR_UNSUPPORTED:
+            groups_ok = False
+            ws = B.decode_workspace(b, False) if Rd else None
+            step()
+        else:
+            raise
+    torch.cuda.synchronize()
+    pkv.pkv_trace_enable(b.pool, True)
+    for _ in range(warmup):
+        flush()
+        step()
+    torch.cuda.synchronize()
+    pkv.pkv_trace_read(b.pool)            # drop the warm-up launches
+    step_ms = run_steps(step, flush, steps, stream)
+    trace = pkv.pkv_trace_read(b.pool)
+    pkv.pkv_trace_enable(b.pool, False)
+    assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
+    res = dict(name=name, w=w, step_ms=step_ms, trace=trace, groups=groups_ok,
+               dec_bytes=decode_bytes(w, b.dec) if Rd else 0,
+               wr_bytes=write_bytes(w, w.num_new_tokens),
+               pre_flops=prefill_flops(w, b.pre) if Rp else 0, Rd=Rd, Rp=Rp)
+
+    if e2e_steps:
+        # end to end through the C ABI from host buffers: slot mapping on the
+        # host, H2D of the step inputs (pinned), kernels, D2H of the outputs
+        q_h = w.q.pin_memory()
+        k_h = w.new_k.pin_memory()
+        v_h = w.new_v.pin_memory()
+        ctx_h = torch.from_numpy(w.context_lens.astype(np.int32)).pin_memory()
+        slots_h = torch.empty(w.num_new_tokens, dtype=torch.int64).pin_memory()
+        out_dh = torch.empty(out_d.shape, dtype=torch.bfloat16).pin_memory()
+        out_ph = torch.empty(out_p.shape, dtype=torch.bfloat16).pin_memory()
+        h2d = (q_h.numel() * 2 + k_h.numel() * 2 + v_h.numel() * 2 + ctx_h.numel() * 4
+               + slots_h.numel() * 8)
+        d2h = out_dh.numel() * 2 + out_ph.numel() * 2
+
+        def e2e_step():
+            slots_h.numpy()[:] = pkv.kv_slot_mapping(b.pool, b.table_host, w.context_lens, w.new_lens)
+            b.q.copy_(q_h, non_blocking=True)
+            b.k_new.copy_(k_h, non_blocking=True)
+            b.v_new.copy_(v_h, non_blocking=True)
+            b.context_lens.copy_(ctx_h, non_blocking=True)
+            b.slots.copy_(slots_h, non_blocking=True)
+            step()
+            if Rd:
+                out_dh.copy_(out_d, non_blocking=True)
+            if Rp:
+                out_ph.copy_(out_p, non_blocking=True)
+            torch.cuda.current_stream().synchronize()
+
+        for _ in range(max(3, warmup)):
+            e2e_step()
+        t0 = time.perf_counter()
+        for _ in range(e2e_steps):
+            e2e_step()
+        t1 = time.perf_counter()
+        res.update(e2e_ms=(t1 - t0) * 1e3 / e2e_steps, h2d=h2d, d2h=d2h)
+    b.close()
+    del b, flush_buf, ws
+    torch.cuda.empty_cache()
+    return res
+
+
+def summarize(res, peaks):
+    hbm, tf_burst, tf_sust, kind = peaks
+    ms = statistics.mean(res["step_ms"])
+    out = {"ms_per_step": ms, "ms_median": statistics.median(res["step_ms"]),
+           "ms_range": [min(res["step_ms"]), max(res["step_ms"])],
+           "kernels": {k: {"launches": n, "avg_us": 1e3 * t / n} for k, (n, t) in res["trace"].items()}}
+    if res["Rd"]:
+        gbs = (res["dec_bytes"] + res["wr_bytes"]) / (ms * 1e-3) / 1e9
+        out.update(decode_hbm_gbs=gbs, decode_frac_of_measured_hbm=gbs / hbm,
+                   decode_frac_of_8tbs=gbs / 8000.0, prefix_pass=res["groups"])
+    if res["Rp"]:
+        tp = res["trace"].get("prefill")
+        if tp:
+            tfs = res["pre_flops"] / (tp[1] / tp[0] * 1e-3) / 1e12
+            out.update(prefill_tflops=tfs, prefill_frac_of_measured_bf16=tfs / tf_burst)
+    return out
+
+
+def reference_arm(args, rank, world):
+    """The fp64 CPU oracle on the host cores, one decode request per step."""
+    import numpy as np
+
+    import oracle
+    from paper_2605_11232_gb300.workloads import make_workload
+
+    if rank != 0:
+        return 0
+    cores = os.cpu_count() or 1
+    w = make_workload(HEADLINE)
+    R = w.num_requests
+    times, nbytes = [], []
+    for k in range(args.warmup + args.steps):
+        r = k % R
+        t0 = time.perf_counter()
+        oracle.request_attention(w, r, threads=cores)
+        dt = time.perf_counter() - t0
+        if k >= args.warmup:
+            times.append(dt)
+            nbytes.append(int(w.context_lens[r]) * kv_row_bytes(w) + 2 * w.num_q_heads * w.head_dim * 2)
+    gbs = sum(nbytes) / sum(times) / 1e9
+    line = {"impl": "reference", "metric": METRIC, "value": gbs, "unit": "GB/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * statistics.mean(times),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": WORKLOAD_DESC[HEADLINE], "sample": "one decode request per step"},
+            "cpu_baseline": {"value": gbs, "unit": "GB/s", "cores": cores, "kind": "oracle",
+                             "sample": "one l8b_decode request per step (all 32 q heads, full context), "
+                                       "fp64 C oracle, threads = host cores"},
+            "e2e": {"value": gbs, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+METRIC = "prefix-cached paged-attn: prefill TFLOP/s & decode HBM GB/s, % of GB300 peak"
+
+
+def cpu_baseline(w_name, budget_s=12.0):
+    """The oracle as it stands on this host: decode requests of the headline
+    workload until about budget_s seconds of work, all host cores."""
+    import oracle
+    from paper_2605_11232_gb300.workloads import make_workload
+    cores = os.cpu_count() or 1
+    w = make_workload(w_name)
+    t0 = time.perf_counter()
+    done, nbytes = 0, 0
+    groups = set()
+    rows = 0
+    for r in range(w.num_requests):
+        oracle.request_attention(w, r, threads=cores)
+        done += 1
+        rows += int(w.context_lens[r]) - w.prefix_len_of(r)
+        if int(w.group_of_req[r]) >= 0:
+            groups.add(int(w.group_of_req[r]))
+        if time.perf_counter() - t0 > budget_s:
+            break
+    dt = time.perf_counter() - t0
+    rows += sum(w.prefix_lens[g] for g in groups)
+    nbytes = rows * kv_row_bytes(w) + 2 * done * w.num_q_heads * w.head_dim * 2
+    return {"value": nbytes / dt / 1e9, "unit": "GB/s", "cores": cores, "kind": "oracle",
+            "sample": f"{done} of {w.num_requests} {w_name} decode requests (all q heads, full "
+                      f"context), fp64 C oracle, {cores} threads, {dt:.1f} s; bytes counted like the "
+                      "GPU metric (shared prefix once)"}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--quick", action="store_true", help="headline workload only")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    rank, world, local = dist_setup(args.gpus)
+    if args.impl == "reference":
+        return reference_arm(args, rank, world)
+
+    import torch
+    torch.cuda.set_device(local)
+    import __graft_entry__
+    if rank == 0:
+        __graft_entry__.build()
+    barrier(world)
+    from paper_2605_11232_gb300 import pkv
+    pkv.load()
+    peaks = load_peaks()
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    t_start = time.time()
+    head = measure_workload(HEADLINE, args.steps, args.warmup, e2e_steps=max(20, args.steps // 4))
+    t_end = time.time()
+    extra = {}
+    if not args.quick:
+        for name in ("l8b_prefill", "qwen_mixed", "l70b_decode"):
+            try:
+                r = measure_workload(name, max(10, args.steps // 10), 3)
+                extra[name] = summarize(r, peaks)
+            except Exception as e:   # report, do not hide
+                extra[name] = {"error": str(e)}
+    clocks.stop()
+
+    w = head["w"]
+    ms_local = statistics.mean(head["step_ms"])
+    ms = max_over_ranks(ms_local, world)
+    step_bytes = head["dec_bytes"] + head["wr_bytes"]
+    total_bytes = sum_over_ranks(step_bytes, world)
+    value = total_bytes / (ms * 1e-3) / 1e9
+    e2e_ms = max_over_ranks(head["e2e_ms"], world)
+    e2e_val = total_bytes / (e2e_ms * 1e-3) / 1e9
+    hbm, tf_burst, tf_sust, pk_kind = peaks
+    # roofline of the dominant kernel (largest share of traced time)
+    trace = head["trace"]
+    dom = max(trace.items(), key=lambda kv: kv[1][1])[0]
+    n_dom, t_dom = trace[dom]
+    avg_ms = t_dom / n_dom
+    if dom == "decode_split":
+        alg = head["dec_bytes"] if not head["groups"] else None
+    elif dom == "kv_cache_write":
+        alg = head["wr_bytes"]
+    else:
+        alg = None
+    if alg is None:   # the split kernel with the prefix pass reads only private rows
+        prefix_rows = sum(w.prefix_lens)
+        alg = head["dec_bytes"] - prefix_rows * kv_row_bytes(w)
+    achieved = alg / (avg_ms * 1e-3) / 1e9
+    traffic = ncu_traffic(dom, HEADLINE)
+    line = {
+        "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": WORKLOAD_DESC[HEADLINE], "global_batch": int(w.num_requests) * world,
+                   "parallelism": f"replicas{world}", "l2": "flushed before every step (256 MiB write), "
+                   "per-step CUDA events", "prefix_pass": head["groups"],
+                   "bytes_per_step": step_bytes},
+        "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                     "frac": achieved / hbm, "peak_kind": pk_kind, "traffic": traffic,
+                     "algorithmic_bytes_per_launch": alg, "avg_launch_us": avg_ms * 1e3},
+        "e2e": {"value": e2e_val, "unit": "GB/s", "h2d_bytes_per_step": head["h2d"],
+                "d2h_bytes_per_step": head["d2h"], "ms_per_step": e2e_ms},
+        "gpu_launches": int(sum(n for n, _ in trace.values())),
+        "clocks": clocks.summary(t_start, t_end),
+        "kernels": {k: {"launches": n, "avg_us": 1e3 * t / n} for k, (n, t) in trace.items()},
+        "headline": summarize(head, peaks),
+        "workloads": extra,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(HEADLINE)
+    elif rank == 0:
+        line["cpu_baseline"] = None
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    barrier(world)
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

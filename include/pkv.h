@@ -212,6 +212,29 @@ int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
                       float scale, const pkv_prefix_groups *groups, void *workspace,
                       size_t workspace_bytes, pkv_stream_t stream);
 
+/* ---- tracing -------------------------------------------------------------- */
+
+/* Per-kernel device time of the launches made while tracing was on. */
+typedef struct {
+    char name[32];       /* "kv_cache_write", "decode_split", "decode_combine",
+                            "decode_prefix", "prefill" */
+    int32_t launches;    /* launches recorded since the last read            */
+    int32_t reserved;
+    double total_ms;     /* sum of CUDA-event durations of those launches    */
+} pkv_kernel_time;
+
+/* Turn per-launch timing on or off for kernels launched through this pool.
+ * While on, every kernel launch is bracketed by a CUDA event pair recorded on
+ * its stream (the observability of Fig. 1: per-stage latency).  Turning it
+ * off synchronises the device and drops unread records. */
+int pkv_trace_enable(pkv_pool_t pool, int32_t enable);
+
+/* Synchronise on the recorded events and report, per kernel, the launches
+ * and their summed duration since the previous read; then clear the records.
+ * out: host array of max_entries; *n_out gets the number filled.
+ * INVALID_ARG if tracing is off. */
+int pkv_trace_read(pkv_pool_t pool, pkv_kernel_time *out, int32_t max_entries, int32_t *n_out);
+
 /* ---- errors --------------------------------------------------------------- */
 
 /* Synchronise `stream`, then read and clear the pool's device error word.

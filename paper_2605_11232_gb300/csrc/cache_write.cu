@@ -38,17 +38,19 @@ __global__ void __launch_bounds__(256) cache_write_kernel(
 
 cudaError_t launch_cache_write(const void *k_new, const void *v_new, const int64_t *slots,
                                int32_t T, void *k_cache, void *v_cache, int32_t Hkv, int32_t d,
-                               int64_t num_slots, int *err, cudaStream_t stream) {
+                               int64_t num_slots, int *err, cudaStream_t stream, Tracer *tr) {
     if (T <= 0) return cudaSuccess;
     const int32_t chunks_per_row = d / 8;
     const int32_t chunks_per_token = Hkv * chunks_per_row;
     const int64_t total = (int64_t)T * chunks_per_token;
     int64_t blocks = (total + 255) / 256;
     if (blocks > 152 * 16) blocks = 152 * 16;
+    if (tr) tr->begin(kKernelCacheWrite, stream);
     cache_write_kernel<<<(unsigned)blocks, 256, 0, stream>>>(
         reinterpret_cast<const uint4 *>(k_new), reinterpret_cast<const uint4 *>(v_new), slots,
         total, chunks_per_token, chunks_per_row, Hkv, reinterpret_cast<uint4 *>(k_cache),
         reinterpret_cast<uint4 *>(v_cache), num_slots, err);
+    if (tr) tr->end(kKernelCacheWrite, stream);
     return cudaGetLastError();
 }
 

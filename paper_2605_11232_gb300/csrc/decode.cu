@@ -433,7 +433,7 @@ DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_
 
 template <int D>
 static cudaError_t launch_decode_t(const DecodeLayout &L, const DecodeArgs &a, int num_sms,
-                                   int32_t num_blocks_pool, cudaStream_t stream) {
+                                   int32_t num_blocks_pool, cudaStream_t stream, Tracer *tr) {
     const size_t smem = (size_t)(L.R + 1) * sizeof(int32_t);
     static bool attr_set = false;
     if (!attr_set) {
@@ -443,19 +443,23 @@ static cudaError_t launch_decode_t(const DecodeLayout &L, const DecodeArgs &a, i
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
+    if (tr) tr->begin(kKernelDecodeSplit, stream);
     decode_split_kernel<D><<<num_sms, kThreads, smem, stream>>>(a, L, num_blocks_pool);
+    if (tr) tr->end(kKernelDecodeSplit, stream);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const int64_t items = (int64_t)L.R * L.Hq;
     const int64_t grid = (items + 7) / 8;
+    if (tr) tr->begin(kKernelDecodeCombine, stream);
     decode_combine_kernel<D><<<(unsigned)grid, 256, 0, stream>>>(a, L);
+    if (tr) tr->end(kKernelDecodeCombine, stream);
     return cudaGetLastError();
 }
 
 cudaError_t launch_decode(const DecodeLayout &L, const DecodeArgs &a, int num_sms,
-                               int32_t num_blocks_pool, cudaStream_t stream) {
-    if (L.d == 128) return launch_decode_t<128>(L, a, num_sms, num_blocks_pool, stream);
-    return launch_decode_t<64>(L, a, num_sms, num_blocks_pool, stream);
+                          int32_t num_blocks_pool, cudaStream_t stream, Tracer *tr) {
+    if (L.d == 128) return launch_decode_t<128>(L, a, num_sms, num_blocks_pool, stream, tr);
+    return launch_decode_t<64>(L, a, num_sms, num_blocks_pool, stream, tr);
 }
 
 }  // namespace pkv

@@ -16,6 +16,62 @@
 
 #include "pkv_internal.h"
 
+namespace pkv {
+const char *const kKernelNames[kNumKernelIds] = {"kv_cache_write", "decode_split", "decode_combine",
+                                                 "decode_prefix", "prefill"};
+}
+
+namespace {
+
+// Records a CUDA event pair around each launch while enabled; times are
+// read (after a synchronize) by pkv_trace_read.
+struct EventTracer final : pkv::Tracer {
+    struct Rec {
+        int kid;
+        cudaEvent_t a, b;
+    };
+    std::vector<Rec> recs;
+    std::vector<cudaEvent_t> spare;
+    cudaEvent_t pending = nullptr;
+    cudaError_t err = cudaSuccess;
+
+    cudaEvent_t get() {
+        if (!spare.empty()) {
+            cudaEvent_t e = spare.back();
+            spare.pop_back();
+            return e;
+        }
+        cudaEvent_t e = nullptr;
+        cudaError_t r = cudaEventCreate(&e);
+        if (r != cudaSuccess && err == cudaSuccess) err = r;
+        return e;
+    }
+    void begin(int, cudaStream_t s) override {
+        pending = get();
+        if (pending) cudaEventRecord(pending, s);
+    }
+    void end(int kid, cudaStream_t s) override {
+        cudaEvent_t b = get();
+        if (!pending || !b) return;
+        cudaEventRecord(b, s);
+        recs.push_back({kid, pending, b});
+        pending = nullptr;
+    }
+    void recycle() {
+        for (auto &r : recs) {
+            spare.push_back(r.a);
+            spare.push_back(r.b);
+        }
+        recs.clear();
+    }
+    ~EventTracer() override {
+        recycle();
+        for (cudaEvent_t e : spare) cudaEventDestroy(e);
+    }
+};
+
+}  // namespace
+
 struct pkv_pool {
     pkv_pool_desc desc;
     void *k_cache = nullptr;
@@ -28,6 +84,7 @@ struct pkv_pool {
     bool tmaps_ready = false;
     CUtensorMap tmap_k;
     CUtensorMap tmap_v;
+    EventTracer *tracer = nullptr;   // non-null while tracing is enabled
 };
 
 namespace {
@@ -166,6 +223,7 @@ int kv_pool_create(const pkv_pool_desc *desc, void *k_cache, void *v_cache, pkv_
 int kv_pool_destroy(pkv_pool_t pool) {
     if (!pool) return ok();
     if (pool->d_err) cudaFree(pool->d_err);
+    delete pool->tracer;
     delete pool;
     return ok();
 }
@@ -290,7 +348,7 @@ int kv_cache_write(pkv_pool_t pool, const void *k_new, const void *v_new,
     cudaError_t e = pkv::launch_cache_write(k_new, v_new, slot_mapping, num_tokens, pool->k_cache,
                                             pool->v_cache, d.num_kv_heads, d.head_dim,
                                             (int64_t)d.num_blocks * 16, pool->d_err,
-                                            static_cast<cudaStream_t>(stream));
+                                            static_cast<cudaStream_t>(stream), pool->tracer);
     if (e != cudaSuccess) return cuda_fail(e, "kv_cache_write launch");
     return ok();
 }
@@ -325,7 +383,7 @@ int paged_attn_prefill(pkv_pool_t pool, const void *q, void *out, float *lse,
     a.scale_log2 = scale * 1.4426950408889634f;
     a.tmap_k = &pool->tmap_k; a.tmap_v = &pool->tmap_v;
     a.err = pool->d_err;
-    cudaError_t e = pkv::launch_prefill(a, static_cast<cudaStream_t>(stream));
+    cudaError_t e = pkv::launch_prefill(a, static_cast<cudaStream_t>(stream), pool->tracer);
     if (e != cudaSuccess) return cuda_fail(e, "paged_attn_prefill launch");
     return ok();
 }
@@ -391,7 +449,7 @@ int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
     a.ws = workspace;
     a.err = pool->d_err;
     cudaError_t e = pkv::launch_decode(L, a, pool->num_sms, d.num_blocks,
-                                       static_cast<cudaStream_t>(stream));
+                                       static_cast<cudaStream_t>(stream), pool->tracer);
     if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode launch");
     return ok();
 }
@@ -408,6 +466,55 @@ int pkv_check_device_errors(pkv_pool_t pool, pkv_stream_t stream, int32_t *code_
     if (e == cudaSuccess) e = cudaMemset(pool->d_err, 0, sizeof(int));
     if (e != cudaSuccess) return cuda_fail(e, "reading the device error word");
     *code_out = v;
+    return ok();
+}
+
+int pkv_trace_enable(pkv_pool_t pool, int32_t enable) {
+    int rc = check_kernel_pool(pool);
+    if (rc != PKV_OK) return rc;
+    if (enable && !pool->tracer) pool->tracer = new EventTracer();
+    if (!enable && pool->tracer) {
+        if ((rc = set_device(pool)) != PKV_OK) return rc;
+        cudaDeviceSynchronize();
+        delete pool->tracer;
+        pool->tracer = nullptr;
+    }
+    return ok();
+}
+
+int pkv_trace_read(pkv_pool_t pool, pkv_kernel_time *out, int32_t max_entries, int32_t *n_out) {
+    int rc = check_kernel_pool(pool);
+    if (rc != PKV_OK) return rc;
+    if (!n_out || max_entries < 0 || (max_entries > 0 && !out))
+        return fail(PKV_ERR_INVALID_ARG, "bad arguments");
+    *n_out = 0;
+    EventTracer *t = pool->tracer;
+    if (!t) return fail(PKV_ERR_INVALID_ARG, "tracing is not enabled");
+    if ((rc = set_device(pool)) != PKV_OK) return rc;
+    if (t->err != cudaSuccess) return cuda_fail(t->err, "trace event");
+    double tot[pkv::kNumKernelIds] = {0};
+    int32_t cnt[pkv::kNumKernelIds] = {0};
+    for (auto &r : t->recs) {
+        cudaError_t e = cudaEventSynchronize(r.b);
+        float ms = 0.f;
+        if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, r.a, r.b);
+        if (e != cudaSuccess) return cuda_fail(e, "reading trace events");
+        tot[r.kid] += ms;
+        cnt[r.kid] += 1;
+    }
+    t->recycle();
+    int32_t n = 0;
+    for (int k = 0; k < pkv::kNumKernelIds; ++k) {
+        if (!cnt[k]) continue;
+        if (n < max_entries) {
+            memset(&out[n], 0, sizeof(out[n]));
+            snprintf(out[n].name, sizeof(out[n].name), "%s", pkv::kKernelNames[k]);
+            out[n].launches = cnt[k];
+            out[n].total_ms = tot[k];
+        }
+        ++n;
+    }
+    *n_out = n < max_entries ? n : max_entries;
     return ok();
 }
 

@@ -8,6 +8,25 @@
 
 namespace pkv {
 
+// Kernels the library launches (names reported by pkv_trace_read).
+enum KernelId : int {
+    kKernelCacheWrite = 0,
+    kKernelDecodeSplit = 1,
+    kKernelDecodeCombine = 2,
+    kKernelDecodePrefix = 3,
+    kKernelPrefill = 4,
+    kNumKernelIds = 5,
+};
+extern const char *const kKernelNames[kNumKernelIds];
+
+// Optional per-launch timing: a CUDA event pair recorded on the launch stream
+// around each kernel (null = tracing off).
+struct Tracer {
+    virtual void begin(int kernel_id, cudaStream_t s) = 0;
+    virtual void end(int kernel_id, cudaStream_t s) = 0;
+    virtual ~Tracer() {}
+};
+
 // Device error word values (a kernel latches the first one with atomicCAS).
 enum : int {
     kDevOk = 0,
@@ -41,7 +60,7 @@ DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_
 
 cudaError_t launch_cache_write(const void *k_new, const void *v_new, const int64_t *slots,
                                int32_t T, void *k_cache, void *v_cache, int32_t Hkv, int32_t d,
-                               int64_t num_slots, int *err, cudaStream_t stream);
+                               int64_t num_slots, int *err, cudaStream_t stream, Tracer *tr);
 
 struct DecodeArgs {
     const void *q;
@@ -65,7 +84,7 @@ struct DecodeArgs {
 };
 
 cudaError_t launch_decode(const DecodeLayout &L, const DecodeArgs &a, int num_sms,
-                          int32_t num_blocks_pool, cudaStream_t stream);
+                          int32_t num_blocks_pool, cudaStream_t stream, Tracer *tr);
 
 struct PrefillArgs {
     const void *q;
@@ -83,6 +102,6 @@ struct PrefillArgs {
     int *err;
 };
 
-cudaError_t launch_prefill(const PrefillArgs &a, cudaStream_t stream);
+cudaError_t launch_prefill(const PrefillArgs &a, cudaStream_t stream, Tracer *tr);
 
 }  // namespace pkv

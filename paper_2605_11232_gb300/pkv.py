@@ -32,7 +32,8 @@ EXPORTS = [
     "kv_pool_create", "kv_pool_destroy", "kv_pool_alloc", "kv_pool_retain", "kv_pool_release",
     "kv_pool_refcount", "kv_pool_num_free", "kv_pool_alloc_sequence", "kv_slot_mapping",
     "kv_cache_write", "paged_attn_prefill", "paged_attn_decode_workspace_size",
-    "paged_attn_decode", "pkv_check_device_errors", "pkv_last_error",
+    "paged_attn_decode", "pkv_trace_enable", "pkv_trace_read", "pkv_check_device_errors",
+    "pkv_last_error",
 ]
 
 
@@ -47,6 +48,11 @@ class PoolDesc(ctypes.Structure):
                 ("num_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
                 ("dtype", ctypes.c_int32), ("reserved", ctypes.c_int32),
                 ("placement_seed", ctypes.c_uint64)]
+
+
+class KernelTime(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char * 32), ("launches", ctypes.c_int32),
+                ("reserved", ctypes.c_int32), ("total_ms", ctypes.c_double)]
 
 
 class PrefixGroups(ctypes.Structure):
@@ -88,6 +94,8 @@ def load(path: str | None = None):
         "paged_attn_decode": [V, V, V, V, V, V, i32, i32, i32, f32,
                               ctypes.POINTER(PrefixGroups), V, sz, V],
         "pkv_check_device_errors": [V, V, P],
+        "pkv_trace_enable": [V, i32],
+        "pkv_trace_read": [V, P, i32, P],
     }
     for name, args in sig.items():
         fn = getattr(lib, name)
@@ -231,6 +239,19 @@ def paged_attn_decode(pool, q, out, lse, context_lens, block_table, scale: float
         ctypes.byref(groups) if groups is not None else None, _dptr(workspace),
         int(workspace.numel() * workspace.element_size()) if workspace is not None else 0,
         _stream(stream)))
+
+
+def pkv_trace_enable(pool, enable: bool = True):
+    _check(load().pkv_trace_enable(pool, 1 if enable else 0))
+
+
+def pkv_trace_read(pool) -> dict:
+    """{kernel name: (launches, total_ms)} since the previous read."""
+    arr = (KernelTime * 8)()
+    n = np.zeros(1, np.int32)
+    _check(load().pkv_trace_read(pool, ctypes.cast(arr, ctypes.c_void_p), 8, _np_ptr(n)))
+    return {arr[i].name.decode(): (int(arr[i].launches), float(arr[i].total_ms))
+            for i in range(int(n[0]))}
 
 
 def pkv_check_device_errors(pool, stream=None) -> int:
