@@ -380,6 +380,7 @@ int paged_attn_prefill(pkv_pool_t pool, const void *q, void *out, float *lse,
     a.block_table = block_table; a.max_blocks = max_blocks;
     a.R = num_requests; a.Hq = num_q_heads; a.Hkv = d.num_kv_heads; a.d = d.head_dim;
     a.max_seqlen_q = max_seqlen_q;
+    a.num_blocks_pool = d.num_blocks;
     a.scale_log2 = scale * 1.4426950408889634f;
     a.tmap_k = &pool->tmap_k; a.tmap_v = &pool->tmap_v;
     a.err = pool->d_err;

@@ -96,6 +96,7 @@ struct PrefillArgs {
     int32_t max_blocks;
     int32_t R, Hq, Hkv, d;
     int32_t max_seqlen_q;
+    int32_t num_blocks_pool;
     float scale_log2;
     const CUtensorMap *tmap_k;  // host copies, passed by value to the kernel
     const CUtensorMap *tmap_v;

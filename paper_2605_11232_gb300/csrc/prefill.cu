@@ -1,5 +1,416 @@
-// prefill.cu -- placeholder until the tcgen05 prefill kernel lands.
+// prefill.cu -- suffix/chunk prefill over a paged, prefix-cached KV cache on
+// the 5th-generation tensor cores (tcgen05, TMEM, TMA).
+//
+// The paper's serving stack reuses the KV blocks of a shared policy prefix and
+// computes only the case-specific suffix (Sec. 5.4; the "enable APC" row of
+// the bottleneck table): every new token attends to the whole cached context
+// plus, causally, to the new tokens before it.  One CTA computes one 128-row
+// tile of (new token, q head) pairs for one kv head: the g q heads of a kv
+// head are packed next to each other (row = token * g + head), so one K/V tile
+// serves all of them (GQA packing).
+//
+// Pipeline (one CTA, 6 warps):
+//   warp 0   TMA producer: for each 128-key tile, 8 paged blocks x (head-dim
+//            halves) of K and of V, each a 16-row x 128-byte box read through
+//            the block table, into a 2-stage ring (128-byte swizzle).
+//   warp 1   MMA issuer (one thread): S = Q K^T into TMEM (double-buffered),
+//            then O += P V with P read from TMEM and V from shared memory.
+//   warps 2-5  softmax: thread = row; S row from TMEM, scale, causal mask,
+//            online max/sum in base 2, P (bf16) written back over S in TMEM;
+//            O is rescaled in TMEM only when the running max grows by more
+//            than 2^8 (otherwise the stale max is kept -- exact, since the same
+//            max normalises O and l).  Epilogue: O / l -> bf16, LSE.
+// Every mbarrier wait is bounded; on a timeout the CTA stops, drains its own
+// TMA copies and MMAs, frees TMEM and latches PKV_ERR_DEVICE_TIMEOUT.
+#include <math.h>
+
+#include "pkv_device.cuh"
 #include "pkv_internal.h"
+#include "tc_ptx.cuh"
+
 namespace pkv {
-cudaError_t launch_prefill(const PrefillArgs &, cudaStream_t, Tracer *) { return cudaErrorNotSupported; }
+
+namespace {
+
+using namespace tc;
+
+constexpr int kThreads = 192;
+constexpr int kRows = 128;            // M of the tile
+constexpr int kKeys = 128;            // keys per tile (N of Q.K^T)
+constexpr uint32_t kTmemCols = 512;   // S0 [0,128) S1 [128,256) O [256, 256+D)
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+constexpr uint64_t kDrainLimitNs = 200000000ull;
+
+template <int D>
+struct Layout {
+    static constexpr int kHalves = D / 64;            // 64-element (128-byte) column halves
+    static constexpr int kHalfBytes = 128 * 128;      // 128 rows x 128 bytes
+    static constexpr int kQ = 0;
+    static constexpr int kTile = kHalves * kHalfBytes;  // one Q, K or V tile
+    static constexpr int kK0 = kQ + kTile;
+    static constexpr int kV0 = kK0 + 2 * kTile;
+    static constexpr int kBar = kV0 + 2 * kTile;
+    // barrier block: k_full[2] v_full[2] kv_empty[2] s_full[2] p_full[2] o_ready done
+    static constexpr int kKFull = kBar + 0, kVFull = kBar + 16, kKvEmpty = kBar + 32;
+    static constexpr int kSFull = kBar + 48, kPFull = kBar + 64, kOReady = kBar + 80;
+    static constexpr int kDone = kBar + 88, kTmemSlot = kBar + 96, kAbort = kBar + 100;
+    static constexpr int kBytes = kBar + 128;
+    static constexpr int kDynSmem = kBytes + 1024;    // room to align the base to 1 KiB
+};
+
+struct KernelParams {
+    const uint16_t *q;
+    uint16_t *out;
+    float *lse;
+    const int32_t *cu_seqlens_q;
+    const int32_t *context_lens;
+    const int32_t *block_table;
+    int32_t max_blocks;
+    int32_t Hq, Hkv, g, tpt;   // tpt: tokens per 128-row tile
+    int32_t num_blocks_pool;
+    float scale_log2;
+    int *err;
+};
+
+// TMEM address of the c-th 32-column chunk of the O accumulator in this
+// warp's lane quarter.
+__device__ __forceinline__ uint32_t o_addr(uint32_t tmem, uint32_t lane_off, int c) {
+    return tmem + lane_off + 256 + c * 32;
+}
+
+__device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile int *abort) {
+    return mbar_wait(bar, parity, abort, kWaitLimitNs);
+}
+
+// Whole-warp wait with a warp-uniform outcome, so that the .sync.aligned
+// tcgen05 instructions after it are reached by all lanes or by none.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int *abort) {
+    return __all_sync(0xffffffffu, wait_bar(bar, parity, abort));
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    prefill_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
+                   const KernelParams p) {
+    using Ly = Layout<D>;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int r = blockIdx.x / p.Hkv, h = blockIdx.x % p.Hkv;
+    const int tile = gridDim.y - 1 - blockIdx.y;      // heaviest tiles first
+    const int cu0 = __ldg(p.cu_seqlens_q + r);
+    const int n_r = __ldg(p.cu_seqlens_q + r + 1) - cu0;
+    const int tok0 = tile * p.tpt;
+    if (tok0 >= n_r) return;
+    const int ntok = min(p.tpt, n_r - tok0);
+    const int L = __ldg(p.context_lens + r);
+    if (L < n_r || L > 16 * p.max_blocks) {
+        if (threadIdx.x == 0) latch_error(p.err, kDevBounds);
+        return;
+    }
+    const int q_pos0 = L - n_r + tok0;     // absolute position of the tile's first token
+    const int kv_end = q_pos0 + ntok;      // keys [0, kv_end) are visible to some row
+    const int nblk = (kv_end + 15) >> 4;
+    const int nkt = (kv_end + kKeys - 1) / kKeys;
+
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                ~uintptr_t(1023));
+    const uint32_t sb = smem_u32(smem);
+    volatile int *abort = reinterpret_cast<volatile int *>(smem + Ly::kAbort);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + Ly::kTmemSlot);
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(sb + Ly::kKFull + 8 * i, 1);
+            mbar_init(sb + Ly::kVFull + 8 * i, 1);
+            mbar_init(sb + Ly::kKvEmpty + 8 * i, 1);
+            mbar_init(sb + Ly::kSFull + 8 * i, 1);
+            mbar_init(sb + Ly::kPFull + 8 * i, 128);
+        }
+        mbar_init(sb + Ly::kOReady, 1);
+        mbar_init(sb + Ly::kDone, 1);
+        *abort = 0;
+        fence_barrier_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+        tmem_relinquish();
+    }
+    // Q tile -> shared memory, K-major with the 128-byte swizzle (16-byte
+    // chunk c of row i goes to chunk c ^ (i % 8) of its 128-byte row).
+    {
+        constexpr int kChunks = D / 8;
+        const int rows_valid = ntok * p.g;
+        for (int idx = threadIdx.x; idx < kRows * kChunks; idx += kThreads) {
+            const int i = idx / kChunks, c = idx % kChunks;
+            uint4 v = make_uint4(0, 0, 0, 0);
+            if (i < rows_valid) {
+                const int tok = i / p.g, hd = i % p.g;
+                v = ldg16(p.q + ((int64_t)(cu0 + tok0 + tok) * p.Hq + h * p.g + hd) * D + c * 8);
+            }
+            const int half = c >> 3, cc = c & 7;
+            *reinterpret_cast<uint4 *>(smem + Ly::kQ + half * Ly::kHalfBytes + i * 128 +
+                                       ((cc ^ (i & 7)) << 4)) = v;
+        }
+        fence_proxy_async_smem();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            prefetch_tmap(&tmk);
+            prefetch_tmap(&tmv);
+            const int32_t *trow = p.block_table + (int64_t)r * p.max_blocks;
+            int issued = 0;
+            for (int j = 0; j < nkt; ++j) {
+                const int s = j & 1;
+                if (j >= 2 && !wait_bar(sb + Ly::kKvEmpty + 8 * s, ((j >> 1) - 1) & 1, abort)) break;
+                const int b0 = j * 8, nb = min(8, nblk - b0);
+                const uint32_t bytes = (uint32_t)nb * Ly::kHalves * 2048u;
+                const uint32_t kdst = sb + Ly::kK0 + s * Ly::kTile;
+                const uint32_t vdst = sb + Ly::kV0 + s * Ly::kTile;
+                int32_t phys[8];
+                for (int b = 0; b < nb; ++b) {
+                    int32_t id = __ldg(trow + b0 + b);
+                    if (id < 0 || id >= p.num_blocks_pool) {
+                        latch_error(p.err, kDevBounds);
+                        id = 0;
+                    }
+                    phys[b] = id;
+                }
+                mbar_arrive_expect_tx(sb + Ly::kKFull + 8 * s, bytes);
+                for (int b = 0; b < nb; ++b)
+                    for (int hf = 0; hf < Ly::kHalves; ++hf)
+                        tma_load_4d(kdst + hf * Ly::kHalfBytes + b * 2048, &tmk, hf * 64, 0, h,
+                                    phys[b], sb + Ly::kKFull + 8 * s);
+                mbar_arrive_expect_tx(sb + Ly::kVFull + 8 * s, bytes);
+                for (int b = 0; b < nb; ++b)
+                    for (int hf = 0; hf < Ly::kHalves; ++hf)
+                        tma_load_4d(vdst + hf * Ly::kHalfBytes + b * 2048, &tmv, hf * 64, 0, h,
+                                    phys[b], sb + Ly::kVFull + 8 * s);
+                issued = j + 1;
+            }
+            // let this CTA's own copies land before its shared memory is released
+            int quiet = 0;
+            for (int j = max(0, issued - 2); j < issued; ++j) {
+                mbar_wait(sb + Ly::kKFull + 8 * (j & 1), (j >> 1) & 1, &quiet, kDrainLimitNs);
+                mbar_wait(sb + Ly::kVFull + 8 * (j & 1), (j >> 1) & 1, &quiet, kDrainLimitNs);
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        const uint32_t id_qk = idesc_bf16_f32(kRows, kKeys, false);
+        const uint32_t id_pv = idesc_bf16_f32(kRows, D, true);
+        const uint32_t o_col = tmem + 256;
+        bool ok = true;
+        auto issue_pv = [&](int jj) -> bool {
+            const int s = jj & 1;
+            if (!warp_wait(sb + Ly::kVFull + 8 * s, (jj >> 1) & 1, abort)) return false;
+            if (!warp_wait(sb + Ly::kPFull + 8 * s, (jj >> 1) & 1, abort)) return false;
+            const uint32_t vbase = sb + Ly::kV0 + s * Ly::kTile;
+            if (jj == nkt - 1) {
+                // keys past the context: p = 0 there, but their V rows may hold
+                // anything (0 * NaN = NaN in the MMA), so clear them
+                const int first = kv_end - jj * kKeys;
+                uint8_t *vs = smem + Ly::kV0 + s * Ly::kTile;
+                for (int row = first + lane; row < kKeys; row += 32)
+                    for (int hf = 0; hf < Ly::kHalves; ++hf) {
+                        uint4 *d4 = reinterpret_cast<uint4 *>(vs + hf * Ly::kHalfBytes + row * 128);
+#pragma unroll
+                        for (int c = 0; c < 8; ++c) d4[c] = make_uint4(0, 0, 0, 0);
+                    }
+                fence_proxy_async_smem();
+                __syncwarp();
+            }
+            tc_fence_after();
+            if (lane == 0) {
+#pragma unroll
+                for (int kk = 0; kk < kKeys / 16; ++kk) {
+                    // V is N-major (head dim contiguous): LBO = stride between the
+                    // 64-wide head-dim halves, SBO = stride between 8-key groups
+                    const uint64_t bdesc = smem_desc_sw128(vbase + kk * 2048, Ly::kHalfBytes, 1024);
+                    mma_ts(o_col, tmem + s * 128 + kk * 8, bdesc, id_pv, (jj > 0 || kk > 0) ? 1u : 0u);
+                }
+                mma_commit(sb + Ly::kKvEmpty + 8 * s);
+                mma_commit(sb + Ly::kOReady);
+            }
+            __syncwarp();
+            return true;
+        };
+        for (int j = 0; j < nkt && ok; ++j) {
+            const int s = j & 1;
+            if (!warp_wait(sb + Ly::kKFull + 8 * s, (j >> 1) & 1, abort)) { ok = false; break; }
+            tc_fence_after();
+            if (lane == 0) {
+                const uint32_t qbase = sb + Ly::kQ, kbase = sb + Ly::kK0 + s * Ly::kTile;
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk) {
+                    const uint32_t off = (kk >> 2) * Ly::kHalfBytes + (kk & 3) * 32;
+                    mma_ss(tmem + s * 128, smem_desc_sw128(qbase + off, 16, 1024),
+                           smem_desc_sw128(kbase + off, 16, 1024), id_qk, kk > 0 ? 1u : 0u);
+                }
+                mma_commit(sb + Ly::kSFull + 8 * s);
+            }
+            __syncwarp();
+            if (j >= 1) ok = issue_pv(j - 1);
+        }
+        if (ok) ok = issue_pv(nkt - 1);
+        // all MMAs issued by this thread must finish before TMEM is freed
+        if (lane == 0) mma_commit(sb + Ly::kDone);
+        __syncwarp();
+        int quiet = 0;
+        mbar_wait(sb + Ly::kDone, 0, &quiet, kDrainLimitNs);
+    } else {
+        // ------------------------------------------------------------ softmax
+        const int quarter = warp & 3;                 // TMEM lanes this warp may touch
+        const int row = quarter * 32 + lane;
+        const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
+        const int rows_valid = ntok * p.g;
+        const bool valid = row < rows_valid;
+        const int tok = row / p.g, hd = row % p.g;
+        const int pos = valid ? q_pos0 + tok : kv_end - 1;
+        float m = -INFINITY, l = 0.f;
+        bool ok = true;
+        for (int j = 0; j < nkt; ++j) {
+            const int b = j & 1;
+            if (!warp_wait(sb + Ly::kSFull + 8 * b, (j >> 1) & 1, abort)) { ok = false; break; }
+            tc_fence_after();
+            uint32_t sr[4][32];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_off + b * 128 + c * 32, sr[c]);
+            tmem_wait_ld();
+            const int kb = j * kKeys;
+            const int lim = pos - kb;                 // keys with column index <= lim are visible
+            float mx = -INFINITY;
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+#pragma unroll
+                for (int e = 0; e < 32; ++e) {
+                    float v = __uint_as_float(sr[c][e]) * p.scale_log2;
+                    v = (c * 32 + e <= lim) ? v : -INFINITY;
+                    sr[c][e] = __float_as_uint(v);
+                    mx = fmaxf(mx, v);
+                }
+            // conditional rescale: keep a stale max unless it grows by > 8 (x256)
+            const float m_new = (mx > m + 8.0f) ? mx : m;
+            const bool grow = (m_new != m) && (j > 0);
+            float alpha = grow ? fast_exp2(m - m_new) : 1.0f;
+            if (j >= 1) {
+                if (!warp_wait(sb + Ly::kOReady, (j - 1) & 1, abort)) { ok = false; break; }
+                tc_fence_after();
+                if (__any_sync(0xffffffffu, grow)) {
+#pragma unroll
+                    for (int c = 0; c < D / 32; ++c) {
+                        uint32_t o[32];
+                        tmem_ld32(o_addr(tmem, lane_off, c), o);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+                        tmem_st32(o_addr(tmem, lane_off, c), o);
+                    }
+                }
+            }
+            m = m_new;
+            float sum = 0.f;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                uint32_t pk[16];
+#pragma unroll
+                for (int e = 0; e < 16; ++e) {
+                    const float p0 = fast_exp2(__uint_as_float(sr[c][2 * e]) - m);
+                    const float p1 = fast_exp2(__uint_as_float(sr[c][2 * e + 1]) - m);
+                    sum += p0 + p1;
+                    pk[e] = pack_bf16x2(p0, p1);
+                }
+                tmem_st16(tmem + lane_off + b * 128 + c * 16, pk);
+            }
+            l = l * alpha + sum;
+            tmem_wait_st();
+            tc_fence_before();
+            mbar_arrive(sb + Ly::kPFull + 8 * b);
+        }
+        if (ok && warp_wait(sb + Ly::kOReady, (nkt - 1) & 1, abort)) {
+            tc_fence_after();
+            const float inv = 1.0f / l;
+            const int64_t orow = ((int64_t)(cu0 + tok0 + tok) * p.Hq + h * p.g + hd);
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t o[32];
+                tmem_ld32(o_addr(tmem, lane_off, c), o);
+                tmem_wait_ld();
+                if (valid) {
+                    uint4 *dst = reinterpret_cast<uint4 *>(p.out + orow * D + c * 32);
+#pragma unroll
+                    for (int v = 0; v < 4; ++v) {
+                        uint4 w;
+                        w.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv, __uint_as_float(o[8 * v + 1]) * inv);
+                        w.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv, __uint_as_float(o[8 * v + 3]) * inv);
+                        w.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv, __uint_as_float(o[8 * v + 5]) * inv);
+                        w.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv, __uint_as_float(o[8 * v + 7]) * inv);
+                        dst[v] = w;
+                    }
+                }
+            }
+            if (valid && p.lse) p.lse[orow] = (m + __log2f(l)) * 0.69314718055994530942f;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+    if (threadIdx.x == 0 && *abort) latch_error(p.err, kDevTimeout);
+}
+
+}  // namespace
+
+cudaError_t launch_prefill(const PrefillArgs &a, cudaStream_t stream, Tracer *tr) {
+    const int g = a.Hq / a.Hkv;
+    KernelParams p{};
+    p.q = static_cast<const uint16_t *>(a.q);
+    p.out = static_cast<uint16_t *>(a.out);
+    p.lse = a.lse;
+    p.cu_seqlens_q = a.cu_seqlens_q;
+    p.context_lens = a.context_lens;
+    p.block_table = a.block_table;
+    p.max_blocks = a.max_blocks;
+    p.Hq = a.Hq; p.Hkv = a.Hkv; p.g = g; p.tpt = kRows / g;
+    p.num_blocks_pool = a.num_blocks_pool;
+    p.scale_log2 = a.scale_log2;
+    p.err = a.err;
+    const int tiles = (a.max_seqlen_q + p.tpt - 1) / p.tpt;
+    if (tiles <= 0 || a.R <= 0) return cudaSuccess;
+    if (tiles > 65535) return cudaErrorInvalidConfiguration;
+    dim3 grid((unsigned)(a.R * a.Hkv), (unsigned)tiles);
+    cudaError_t e;
+    if (tr) tr->begin(kKernelPrefill, stream);
+    if (a.d == 128) {
+        static bool attr = false;
+        if (!attr) {
+            e = cudaFuncSetAttribute(prefill_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     Layout<128>::kDynSmem);
+            if (e != cudaSuccess) return e;
+            attr = true;
+        }
+        prefill_kernel<128><<<grid, kThreads, Layout<128>::kDynSmem, stream>>>(*a.tmap_k, *a.tmap_v, p);
+    } else {
+        static bool attr = false;
+        // the d = 64 tile is smaller; ask for the d = 128 footprint anyway so
+        // one CTA owns an SM (its 512 TMEM columns never wait on a neighbour)
+        if (!attr) {
+            e = cudaFuncSetAttribute(prefill_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     Layout<128>::kDynSmem);
+            if (e != cudaSuccess) return e;
+            attr = true;
+        }
+        prefill_kernel<64><<<grid, kThreads, Layout<128>::kDynSmem, stream>>>(*a.tmap_k, *a.tmap_v, p);
+    }
+    if (tr) tr->end(kKernelPrefill, stream);
+    return cudaGetLastError();
+}
+
 }  // namespace pkv

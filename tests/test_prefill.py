@@ -1,0 +1,182 @@
+"""paged_attn_prefill against the fp64 oracle (GPU).
+
+Suffix (or chunk) tokens attend to the whole cached context (shared prefix
+included) and causally to the new tokens.  Tolerance as for decode: max abs
+1e-2, mean abs 1e-3 over the compared elements; LSE within 1e-3.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2605_11232_gb300 import batch as B
+from paper_2605_11232_gb300 import pkv
+from paper_2605_11232_gb300.workloads import make_workload
+
+from _lib import need_gpu
+
+pytestmark = pytest.mark.gpu
+
+MAX_ABS, MEAN_ABS, LSE_ABS = 1e-2, 1e-3, 1e-3
+
+
+def _f64(t):
+    return t.detach().float().cpu().numpy().astype(np.float64)
+
+
+def run_prefill(b, with_lse=True):
+    w = b.w
+    rows = B.new_token_rows(w, b.pre)
+    n = rows.stop - rows.start
+    B.run_write(b)
+    out = torch.full((n, w.num_q_heads, w.head_dim), float("nan"), dtype=torch.bfloat16, device="cuda")
+    lse = torch.full((n, w.num_q_heads), float("nan"), dtype=torch.float32, device="cuda") if with_lse else None
+    B.run_prefill(b, out, lse)
+    assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
+    return out, lse
+
+
+def compare(b, out, lse, reqs, rows_per_req=None, threads=16, seed=0):
+    """Compare every (or a sample of) query rows of the given requests."""
+    w = b.w
+    rng = np.random.default_rng(seed)
+    base = int(w.cu_new[b.pre.start])
+    errs, lerrs = [], []
+    for r in reqs:
+        S = int(w.new_lens[r])
+        if rows_per_req is None or rows_per_req >= S:
+            sel = list(range(S))
+            ref_o, ref_l = oracle.request_attention(w, r, threads=threads)
+        else:
+            sel = sorted({0, S - 1, *rng.choice(S, rows_per_req - 2, replace=False).tolist()})
+            ref_o, ref_l = oracle.request_attention(w, r, threads=threads, rows=sel)
+        off = int(w.cu_new[r]) - base
+        got = _f64(out[[off + i for i in sel]])
+        errs.append(np.abs(got - ref_o).ravel())
+        if lse is not None:
+            lerrs.append(np.abs(_f64(lse[[off + i for i in sel]]) - ref_l).ravel())
+    e = np.concatenate(errs)
+    assert np.isfinite(e).all()
+    assert e.max() <= MAX_ABS and e.mean() <= MEAN_ABS, (e.max(), e.mean())
+    if lerrs:
+        le = np.concatenate(lerrs)
+        assert le.max() <= LSE_ABS, le.max()
+
+
+def test_tiny_prefill_all_rows():
+    """d = 64, g = 4: 4 suffixes (32/48/64/96) over a shared 256-token prefix."""
+    need_gpu()
+    w = make_workload("tiny")
+    b = B.build_batch(w, poison=True)
+    out, lse = run_prefill(b)
+    compare(b, out, lse, range(w.num_requests))
+    b.close()
+
+
+@pytest.mark.parametrize("Hq,Hkv,d,ctx,new", [
+    (8, 2, 128, [1, 17, 130, 300], [1, 17, 130, 100]),      # no prefix, causal from 0
+    (7, 1, 128, [40, 257], [40, 129]),                        # g = 7: 18 tokens per tile
+    (64, 8, 128, [200, 33], [50, 33]),                        # g = 8: 16 tokens per tile
+    (4, 4, 64, [70, 500], [3, 250]),                          # g = 1 (MHA), d = 64
+    (16, 1, 128, [129, 128], [129, 1]),                       # g = 16
+])
+def test_prefill_shapes_all_rows(Hq, Hkv, d, ctx, new):
+    need_gpu()
+    R = len(ctx)
+    w = make_workload("custom", custom=dict(Hq=Hq, Hkv=Hkv, d=d, prefix_lens=[], group=[-1] * R,
+                                          cached=[c - n for c, n in zip(ctx, new)], new=new,
+                                          decode=[False] * R))
+    b = B.build_batch(w, poison=True)
+    out, lse = run_prefill(b)
+    compare(b, out, lse, range(R))
+    b.close()
+
+
+def test_l8b_prefill_scaled_sampled_rows():
+    """4 requests of the Llama-3-8B suffix-prefill workload (full 4096 prefix)."""
+    need_gpu()
+    w = make_workload("l8b_prefill", scale_requests=0.125)
+    b = B.build_batch(w, poison=True)
+    out, lse = run_prefill(b)
+    compare(b, out, lse, range(w.num_requests), rows_per_req=24)
+    b.close()
+
+
+@pytest.mark.parametrize("name", ["l8b_prefill", "qwen_mixed"])
+def test_prefill_full_size_sampled(name):
+    """Full-size batch (the benchmark's call); sampled rows of 4 requests vs
+    the oracle and no NaN anywhere in the output."""
+    need_gpu()
+    w = make_workload(name)
+    b = B.build_batch(w, poison=True)
+    out, lse = run_prefill(b)
+    assert torch.isfinite(out.float()).all() and torch.isfinite(lse).all()
+    reqs = list(range(b.pre.start, b.pre.stop))
+    pick = sorted({reqs[0], reqs[-1], reqs[len(reqs) // 2],
+                   reqs[int(np.argmax(w.cached_lens[b.pre]))]})
+    compare(b, out, lse, pick, rows_per_req=12)
+    b.close()
+
+
+def test_prefill_last_row_equals_decode():
+    """The last prefill row of a request attends to exactly what a decode query
+    at that position attends to: the two kernels agree within tolerance."""
+    need_gpu()
+    w = make_workload("tiny")
+    b = B.build_batch(w, poison=True)
+    out, lse = run_prefill(b)
+    wd = make_workload("custom", seed=w.seed, custom=dict(
+        Hq=8, Hkv=2, d=64, prefix_lens=[256], group=[0] * 4,
+        cached=list(w.cached_lens + w.new_lens - 1), new=[1] * 4, decode=[True] * 4, num_blocks=64))
+    # same K/V and query rows as the prefill batch's last tokens
+    wd.prefix_k, wd.prefix_v = w.prefix_k, w.prefix_v
+    parts_k, parts_v, q = [], [], []
+    for r in range(4):
+        a, e = int(w.cu_new[r]), int(w.cu_new[r + 1])
+        parts_k.append(torch.cat([w.priv_k[w.priv_off[r]:w.priv_off[r + 1]], w.new_k[a:e - 1]]))
+        parts_v.append(torch.cat([w.priv_v[w.priv_off[r]:w.priv_off[r + 1]], w.new_v[a:e - 1]]))
+        q.append(w.q[e - 1:e])
+    wd.priv_k, wd.priv_v = torch.cat(parts_k), torch.cat(parts_v)
+    wd.priv_off = np.concatenate([[0], np.cumsum([len(x) for x in parts_k])])
+    wd.new_k = torch.cat([w.new_k[int(w.cu_new[r + 1]) - 1:int(w.cu_new[r + 1])] for r in range(4)])
+    wd.new_v = torch.cat([w.new_v[int(w.cu_new[r + 1]) - 1:int(w.cu_new[r + 1])] for r in range(4)])
+    wd.q = torch.cat(q)
+    bd = B.build_batch(wd, poison=True)
+    B.run_write(bd)
+    od = torch.empty((4, 8, 64), dtype=torch.bfloat16, device="cuda")
+    ws = B.decode_workspace(bd, False)
+    B.run_decode(bd, od, None, ws, False)
+    last = [int(w.cu_new[r + 1]) - 1 for r in range(4)]
+    diff = (out[last].float() - od.float()).abs()
+    assert diff.max().item() <= 2e-2
+    b.close(); bd.close()
+
+
+def test_prefill_placement_invariance_bit_exact():
+    need_gpu()
+    w = make_workload("l8b_prefill", scale_requests=0.0625)
+    outs = []
+    for seed in (0, 99):
+        b = B.build_batch(w, poison=True, placement_seed=seed)
+        o, l = run_prefill(b)
+        outs.append((o.cpu(), l.cpu()))
+        b.close()
+    assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
+
+
+def test_prefill_causality_future_keys_ignored():
+    """Changing the K/V of the last new token changes no earlier row."""
+    need_gpu()
+    w = make_workload("tiny")
+    b = B.build_batch(w, poison=True)
+    o1, l1 = run_prefill(b)
+    for r in range(w.num_requests):
+        t = int(w.cu_new[r + 1]) - 1
+        b.k_new[t] = 50.0
+        b.v_new[t] = -7.0
+    o2, l2 = run_prefill(b)
+    for r in range(w.num_requests):
+        a, e = int(w.cu_new[r]), int(w.cu_new[r + 1])
+        assert torch.equal(o1[a:e - 1], o2[a:e - 1]) and torch.equal(l1[a:e - 1], l2[a:e - 1])
+        assert not torch.equal(o1[e - 1], o2[e - 1])
+    b.close()
