@@ -269,7 +269,17 @@ def measure_workload(name, steps, warmup, use_groups=True, e2e_steps=0):
     trace = pkv.pkv_trace_read(b.pool)
     pkv.pkv_trace_enable(b.pool, False)
     assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
-    res = dict(name=name, w=w, step_ms=step_ms, trace=trace, groups=groups_ok,
+    # algorithmic bytes each decode kernel is responsible for
+    kb = {"kv_cache_write": write_bytes(w, w.num_new_tokens)}
+    if Rd:
+        rows_priv = sum(int(w.context_lens[r]) - w.prefix_len_of(r) for r in range(b.dec.start, b.dec.stop))
+        used = {int(w.group_of_req[r]) for r in range(b.dec.start, b.dec.stop)} - {-1}
+        rows_pre = sum(w.prefix_lens[gi] for gi in used)
+        qo = Rd * w.num_q_heads * w.head_dim * 2
+        kb["decode_split"] = (rows_priv + (0 if groups_ok else rows_pre)) * kv_row_bytes(w) + qo
+        kb["decode_prefix"] = rows_pre * kv_row_bytes(w) + qo if groups_ok else 0
+        kb["decode_combine"] = qo
+    res = dict(name=name, w=w, step_ms=step_ms, trace=trace, groups=groups_ok, kernel_bytes=kb,
                dec_bytes=decode_bytes(w, b.dec) if Rd else 0,
                wr_bytes=write_bytes(w, w.num_new_tokens),
                pre_flops=prefill_flops(w, b.pre) if Rp else 0, Rd=Rd, Rp=Rp)
@@ -453,16 +463,8 @@ def main():
     dom = max(trace.items(), key=lambda kv: kv[1][1])[0]
     n_dom, t_dom = trace[dom]
     avg_ms = t_dom / n_dom
-    if dom == "decode_split":
-        alg = head["dec_bytes"] if not head["groups"] else None
-    elif dom == "kv_cache_write":
-        alg = head["wr_bytes"]
-    else:
-        alg = None
-    if alg is None:   # the split kernel with the prefix pass reads only private rows
-        prefix_rows = sum(w.prefix_lens)
-        alg = head["dec_bytes"] - prefix_rows * kv_row_bytes(w)
-    achieved = alg / (avg_ms * 1e-3) / 1e9
+    alg = head["kernel_bytes"].get(dom)
+    achieved = alg / (avg_ms * 1e-3) / 1e9 if alg else None
     traffic = ncu_traffic(dom, HEADLINE)
     line = {
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
@@ -473,7 +475,7 @@ def main():
                    "per-step CUDA events", "prefix_pass": head["groups"],
                    "bytes_per_step": step_bytes},
         "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                     "frac": achieved / hbm, "peak_kind": pk_kind, "traffic": traffic,
+                     "frac": achieved / hbm if achieved else None, "peak_kind": pk_kind, "traffic": traffic,
                      "algorithmic_bytes_per_launch": alg, "avg_launch_us": avg_ms * 1e3},
         "e2e": {"value": e2e_val, "unit": "GB/s", "h2d_bytes_per_step": head["h2d"],
                 "d2h_bytes_per_step": head["d2h"], "ms_per_step": e2e_ms},

@@ -413,13 +413,32 @@ __global__ void __launch_bounds__(256) decode_combine_kernel(DecodeArgs a, Decod
 }  // namespace
 
 DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_t max_blocks,
-                           int32_t num_groups, int32_t max_group_blocks) {
+                           int32_t num_groups, int32_t max_group_blocks, int32_t max_group_members,
+                           int32_t num_sms) {
     DecodeLayout L{};
     L.R = R; L.Hq = Hq; L.Hkv = Hkv; L.d = d; L.g = Hq / Hkv;
-    L.prefix_blocks_per_part = 64;
+    L.prefix_blocks_per_part = 8;
     L.prefix_parts = 0;
-    if (num_groups > 0 && max_group_blocks > 0)
+    if (num_groups > 0 && max_group_blocks > 0 && max_group_members > 0) {
+        // Key splits of the prefix pass: one CTA per (group, kv head, member
+        // tile, split), one CTA per SM.  Pick the split count that minimises
+        // waves x (per-CTA set-up + key tiles per CTA), set-up ~ 2 key tiles.
+        const int tpt = 128 / L.g;
+        const int64_t tiles = (int64_t)num_groups * Hkv * ((max_group_members + tpt - 1) / tpt);
+        const int sms = num_sms > 0 ? num_sms : 148;
+        const int key_tiles = (max_group_blocks + 7) / 8;
+        int best = 1;
+        double best_t = 1e30;
+        for (int sp = 1; sp <= kMaxPrefixParts && sp <= key_tiles; ++sp) {
+            const int per = (key_tiles + sp - 1) / sp;
+            const double waves = (double)((tiles * sp + sms - 1) / sms);
+            const double t = waves * (2.0 + per);
+            if (t < best_t - 1e-9) { best_t = t; best = sp; }
+        }
+        const int per_tiles = (key_tiles + best - 1) / best;
+        L.prefix_blocks_per_part = per_tiles * 8;
         L.prefix_parts = (max_group_blocks + L.prefix_blocks_per_part - 1) / L.prefix_blocks_per_part;
+    }
     L.parts_per_head = L.prefix_parts + kMaxPrivateParts;
     const size_t slots = (size_t)R * Hq * L.parts_per_head;
     auto up = [](size_t x) { return (x + 255) & ~(size_t)255; };
@@ -442,6 +461,10 @@ static cudaError_t launch_decode_t(const DecodeLayout &L, const DecodeArgs &a, i
                                              (kMaxRequestsPlan + 1) * (int)sizeof(int32_t));
         if (e != cudaSuccess) return e;
         attr_set = true;
+    }
+    if (L.prefix_parts > 0 && a.num_groups > 0) {
+        cudaError_t e = launch_decode_prefix(L, a, num_blocks_pool, stream, tr);
+        if (e != cudaSuccess) return e;
     }
     if (tr) tr->begin(kKernelDecodeSplit, stream);
     decode_split_kernel<D><<<num_sms, kThreads, smem, stream>>>(a, L, num_blocks_pool);

@@ -7,6 +7,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <climits>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -396,8 +397,10 @@ int paged_attn_decode_workspace_size(pkv_pool_t pool, int32_t num_requests, int3
         return fail(PKV_ERR_INVALID_ARG, "bad arguments");
     const int32_t G = groups ? groups->num_groups : 0;
     const int32_t mgb = groups ? groups->max_group_blocks : 0;
+    const int32_t mgm = groups ? groups->max_group_members : 0;
     pkv::DecodeLayout L = pkv::decode_layout(num_requests, num_q_heads, pool->desc.num_kv_heads,
-                                             pool->desc.head_dim, max_blocks, G, mgb);
+                                             pool->desc.head_dim, max_blocks, G, mgb, mgm,
+                                             pool->num_sms);
     *bytes_out = L.total;
     return ok();
 }
@@ -420,22 +423,25 @@ int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
     if (num_requests == 0) return ok();
     if (!q || !out || !context_lens || !block_table) return fail(PKV_ERR_INVALID_ARG, "NULL buffer");
     if (!aligned16(q) || !aligned16(out)) return fail(PKV_ERR_INVALID_ARG, "misaligned q/out");
-    int32_t G = 0, mgb = 0;
+    int32_t G = 0, mgb = 0, mgm = 0;
     if (groups && groups->num_groups > 0) {
         G = groups->num_groups;
         mgb = groups->max_group_blocks;
+        mgm = groups->max_group_members;
         if (!groups->group_start || !groups->member_req || !groups->group_blocks ||
-            !groups->group_of_req || mgb < 0 || groups->max_group_members < 0)
+            !groups->group_of_req || mgb < 0 || mgm < 0)
             return fail(PKV_ERR_INVALID_ARG, "incomplete prefix-group descriptor");
-        return fail(PKV_ERR_UNSUPPORTED, "prefix-shared decode pass not built yet");
+        if (mgb > max_blocks) return fail(PKV_ERR_INVALID_ARG, "max_group_blocks exceeds the table width");
+        if ((int64_t)G * d.num_kv_heads > INT32_MAX) return fail(PKV_ERR_UNSUPPORTED, "too many groups");
     }
     pkv::DecodeLayout L = pkv::decode_layout(num_requests, num_q_heads, d.num_kv_heads, d.head_dim,
-                                             max_blocks, G, mgb);
+                                             max_blocks, G, mgb, mgm, pool->num_sms);
     if (!workspace || workspace_bytes < L.total)
         return fail(PKV_ERR_WORKSPACE, "workspace of %zu bytes needed", L.total);
     if (reinterpret_cast<uintptr_t>(workspace) & 255)
         return fail(PKV_ERR_WORKSPACE, "workspace must be 256-byte aligned");
     if ((rc = set_device(pool)) != PKV_OK) return rc;
+    if (L.prefix_parts > 0 && (rc = build_tmaps(pool)) != PKV_OK) return rc;
     pkv::DecodeArgs a{};
     a.q = q; a.out = out; a.lse = lse;
     a.context_lens = context_lens; a.block_table = block_table; a.max_blocks = max_blocks;
@@ -449,6 +455,8 @@ int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
     }
     a.ws = workspace;
     a.err = pool->d_err;
+    a.tmap_k = &pool->tmap_k;
+    a.tmap_v = &pool->tmap_v;
     cudaError_t e = pkv::launch_decode(L, a, pool->num_sms, d.num_blocks,
                                        static_cast<cudaStream_t>(stream), pool->tracer);
     if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode launch");

@@ -56,7 +56,8 @@ struct DecodeLayout {
 };
 
 DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_t max_blocks,
-                           int32_t num_groups, int32_t max_group_blocks);
+                           int32_t num_groups, int32_t max_group_blocks, int32_t max_group_members,
+                           int32_t num_sms);
 
 cudaError_t launch_cache_write(const void *k_new, const void *v_new, const int64_t *slots,
                                int32_t T, void *k_cache, void *v_cache, int32_t Hkv, int32_t d,
@@ -81,6 +82,8 @@ struct DecodeArgs {
     const int32_t *group_of_req;
     void *ws;
     int *err;
+    const CUtensorMap *tmap_k;   // needed by the shared-prefix pass
+    const CUtensorMap *tmap_v;
 };
 
 cudaError_t launch_decode(const DecodeLayout &L, const DecodeArgs &a, int num_sms,
@@ -104,5 +107,11 @@ struct PrefillArgs {
 };
 
 cudaError_t launch_prefill(const PrefillArgs &a, cudaStream_t stream, Tracer *tr);
+
+// Shared-prefix pass of decode (tcgen05 tile kernel in prefix mode): partials
+// of every group member over its group's prefix blocks, split in key ranges of
+// L.prefix_blocks_per_part blocks, into part slots [0, L.prefix_parts).
+cudaError_t launch_decode_prefix(const DecodeLayout &L, const DecodeArgs &a,
+                                 int32_t num_blocks_pool, cudaStream_t stream, Tracer *tr);
 
 }  // namespace pkv

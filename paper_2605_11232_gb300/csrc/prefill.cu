@@ -70,6 +70,15 @@ struct KernelParams {
     int32_t num_blocks_pool;
     float scale_log2;
     int *err;
+    // shared-prefix decode pass only
+    const int32_t *group_start;
+    const int32_t *member_req;
+    const int32_t *group_blocks;
+    int32_t num_requests;       // decode batch size (member ids must be below it)
+    int32_t blocks_per_part;    // prefix blocks per key split
+    int32_t parts_per_head;     // partial slots per (request, q head)
+    float *o_part;              // [R*Hq*parts][D] unnormalised O
+    float2 *ml_part;            // [R*Hq*parts] (running max (base 2), sum)
 };
 
 // TMEM address of the c-th 32-column chunk of the O accumulator in this
@@ -88,28 +97,79 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
     return __all_sync(0xffffffffu, wait_bar(bar, parity, abort));
 }
 
-template <int D>
+// PREFIX = false: suffix prefill.  CTA (request r, kv head h, token tile);
+//   row i = token (i / g) of the tile, q head h*g + i % g; keys 0 .. pos(i).
+// PREFIX = true: shared-prefix pass of decode.  CTA (group, kv head, member
+//   tile, key split); row i = member request (i / g) of the tile; keys = the
+//   split's range of the group's prefix blocks (read through the first
+//   member's table row), all visible; writes unnormalised partials.
+template <int D, bool PREFIX>
 __global__ void __launch_bounds__(kThreads, 1)
-    prefill_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
-                   const KernelParams p) {
+    attn_tile_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
+                     const KernelParams p) {
     using Ly = Layout<D>;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int r = blockIdx.x / p.Hkv, h = blockIdx.x % p.Hkv;
-    const int tile = gridDim.y - 1 - blockIdx.y;      // heaviest tiles first
-    const int cu0 = __ldg(p.cu_seqlens_q + r);
-    const int n_r = __ldg(p.cu_seqlens_q + r + 1) - cu0;
-    const int tok0 = tile * p.tpt;
-    if (tok0 >= n_r) return;
-    const int ntok = min(p.tpt, n_r - tok0);
-    const int L = __ldg(p.context_lens + r);
-    if (L < n_r || L > 16 * p.max_blocks) {
-        if (threadIdx.x == 0) latch_error(p.err, kDevBounds);
-        return;
+    const int h = blockIdx.x % p.Hkv;
+    int rows_valid, nblk, kv_end, q_pos0 = 0, blk_off = 0, cu0 = 0, tok0 = 0, m0 = 0;
+    const int32_t *trow;
+    if constexpr (!PREFIX) {
+        const int r = blockIdx.x / p.Hkv;
+        const int tile = gridDim.y - 1 - blockIdx.y;      // heaviest tiles first
+        cu0 = __ldg(p.cu_seqlens_q + r);
+        const int n_r = __ldg(p.cu_seqlens_q + r + 1) - cu0;
+        tok0 = tile * p.tpt;
+        if (tok0 >= n_r) return;
+        const int ntok = min(p.tpt, n_r - tok0);
+        const int L = __ldg(p.context_lens + r);
+        if (L < n_r || L > 16 * p.max_blocks) {
+            if (threadIdx.x == 0) latch_error(p.err, kDevBounds);
+            return;
+        }
+        q_pos0 = L - n_r + tok0;          // absolute position of the tile's first token
+        kv_end = q_pos0 + ntok;           // keys [0, kv_end) are visible to some row
+        nblk = (kv_end + 15) >> 4;
+        rows_valid = ntok * p.g;
+        trow = p.block_table + (int64_t)r * p.max_blocks;
+    } else {
+        const int grp = blockIdx.x / p.Hkv;
+        const int gs = __ldg(p.group_start + grp);
+        const int nm = __ldg(p.group_start + grp + 1) - gs;
+        const int mt0 = blockIdx.y * p.tpt;
+        if (mt0 >= nm) return;
+        const int gb = __ldg(p.group_blocks + grp);
+        blk_off = blockIdx.z * p.blocks_per_part;
+        if (blk_off >= gb) return;
+        if (gb > p.max_blocks) {
+            if (threadIdx.x == 0) latch_error(p.err, kDevBounds);
+            return;
+        }
+        nblk = min(p.blocks_per_part, gb - blk_off);
+        kv_end = nblk * 16;
+        rows_valid = min(p.tpt, nm - mt0) * p.g;
+        m0 = gs + mt0;
+        // every member id of this tile (and the first member, whose table row
+        // names the prefix blocks) must be a request of the batch
+        bool ids_ok = true;
+        const int r_first = __ldg(p.member_req + gs);
+        if (r_first < 0 || r_first >= p.num_requests) ids_ok = false;
+        for (int i = 0; i < rows_valid; i += p.g) {
+            const int rm = __ldg(p.member_req + m0 + i / p.g);
+            if (rm < 0 || rm >= p.num_requests) ids_ok = false;
+        }
+        if (!ids_ok) {
+            if (threadIdx.x == 0) latch_error(p.err, kDevBounds);
+            return;
+        }
+        trow = p.block_table + (int64_t)r_first * p.max_blocks;
     }
-    const int q_pos0 = L - n_r + tok0;     // absolute position of the tile's first token
-    const int kv_end = q_pos0 + ntok;      // keys [0, kv_end) are visible to some row
-    const int nblk = (kv_end + 15) >> 4;
     const int nkt = (kv_end + kKeys - 1) / kKeys;
+    // global q row of tile row i (decode q is [R][Hq][D], prefill q is [T][Hq][D])
+    auto q_row = [&](int i) -> int64_t {
+        if constexpr (PREFIX)
+            return (int64_t)__ldg(p.member_req + m0 + i / p.g) * p.Hq + h * p.g + i % p.g;
+        else
+            return (int64_t)(cu0 + tok0 + i / p.g) * p.Hq + h * p.g + i % p.g;
+    };
 
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -139,14 +199,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     // chunk c of row i goes to chunk c ^ (i % 8) of its 128-byte row).
     {
         constexpr int kChunks = D / 8;
-        const int rows_valid = ntok * p.g;
         for (int idx = threadIdx.x; idx < kRows * kChunks; idx += kThreads) {
             const int i = idx / kChunks, c = idx % kChunks;
             uint4 v = make_uint4(0, 0, 0, 0);
-            if (i < rows_valid) {
-                const int tok = i / p.g, hd = i % p.g;
-                v = ldg16(p.q + ((int64_t)(cu0 + tok0 + tok) * p.Hq + h * p.g + hd) * D + c * 8);
-            }
+            if (i < rows_valid) v = ldg16(p.q + q_row(i) * D + c * 8);
             const int half = c >> 3, cc = c & 7;
             *reinterpret_cast<uint4 *>(smem + Ly::kQ + half * Ly::kHalfBytes + i * 128 +
                                        ((cc ^ (i & 7)) << 4)) = v;
@@ -163,7 +219,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             prefetch_tmap(&tmk);
             prefetch_tmap(&tmv);
-            const int32_t *trow = p.block_table + (int64_t)r * p.max_blocks;
             int issued = 0;
             for (int j = 0; j < nkt; ++j) {
                 const int s = j & 1;
@@ -174,7 +229,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t vdst = sb + Ly::kV0 + s * Ly::kTile;
                 int32_t phys[8];
                 for (int b = 0; b < nb; ++b) {
-                    int32_t id = __ldg(trow + b0 + b);
+                    int32_t id = __ldg(trow + blk_off + b0 + b);
                     if (id < 0 || id >= p.num_blocks_pool) {
                         latch_error(p.err, kDevBounds);
                         id = 0;
@@ -268,10 +323,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int quarter = warp & 3;                 // TMEM lanes this warp may touch
         const int row = quarter * 32 + lane;
         const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
-        const int rows_valid = ntok * p.g;
         const bool valid = row < rows_valid;
-        const int tok = row / p.g, hd = row % p.g;
-        const int pos = valid ? q_pos0 + tok : kv_end - 1;
+        // last visible key (tile-local numbering of the item's key range)
+        const int pos = (!PREFIX && valid) ? q_pos0 + row / p.g : kv_end - 1;
         float m = -INFINITY, l = 0.f;
         bool ok = true;
         for (int j = 0; j < nkt; ++j) {
@@ -334,27 +388,45 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (ok && warp_wait(sb + Ly::kOReady, (nkt - 1) & 1, abort)) {
             tc_fence_after();
-            const float inv = 1.0f / l;
-            const int64_t orow = ((int64_t)(cu0 + tok0 + tok) * p.Hq + h * p.g + hd);
+            const int64_t orow = valid ? q_row(row) : 0;
+            if constexpr (!PREFIX) {
+                const float inv = 1.0f / l;
 #pragma unroll
-            for (int c = 0; c < D / 32; ++c) {
-                uint32_t o[32];
-                tmem_ld32(o_addr(tmem, lane_off, c), o);
-                tmem_wait_ld();
-                if (valid) {
-                    uint4 *dst = reinterpret_cast<uint4 *>(p.out + orow * D + c * 32);
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t o[32];
+                    tmem_ld32(o_addr(tmem, lane_off, c), o);
+                    tmem_wait_ld();
+                    if (valid) {
+                        uint4 *dst = reinterpret_cast<uint4 *>(p.out + orow * D + c * 32);
 #pragma unroll
-                    for (int v = 0; v < 4; ++v) {
-                        uint4 w;
-                        w.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv, __uint_as_float(o[8 * v + 1]) * inv);
-                        w.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv, __uint_as_float(o[8 * v + 3]) * inv);
-                        w.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv, __uint_as_float(o[8 * v + 5]) * inv);
-                        w.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv, __uint_as_float(o[8 * v + 7]) * inv);
-                        dst[v] = w;
+                        for (int v = 0; v < 4; ++v) {
+                            uint4 w;
+                            w.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv, __uint_as_float(o[8 * v + 1]) * inv);
+                            w.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv, __uint_as_float(o[8 * v + 3]) * inv);
+                            w.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv, __uint_as_float(o[8 * v + 5]) * inv);
+                            w.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv, __uint_as_float(o[8 * v + 7]) * inv);
+                            dst[v] = w;
+                        }
                     }
                 }
+                if (valid && p.lse) p.lse[orow] = (m + __log2f(l)) * 0.69314718055994530942f;
+            } else {
+                // unnormalised partial of key split blockIdx.z, merged by the combine
+                const int64_t slot = orow * p.parts_per_head + blockIdx.z;
+#pragma unroll
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t o[32];
+                    tmem_ld32(o_addr(tmem, lane_off, c), o);
+                    tmem_wait_ld();
+                    if (valid) {
+                        uint4 *dst = reinterpret_cast<uint4 *>(p.o_part + slot * D + c * 32);
+#pragma unroll
+                        for (int v = 0; v < 8; ++v)
+                            dst[v] = make_uint4(o[4 * v], o[4 * v + 1], o[4 * v + 2], o[4 * v + 3]);
+                    }
+                }
+                if (valid) p.ml_part[slot] = make_float2(m, l);
             }
-            if (valid && p.lse) p.lse[orow] = (m + __log2f(l)) * 0.69314718055994530942f;
         }
     }
     tc_fence_before();
@@ -367,6 +439,23 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 }  // namespace
+
+template <int D, bool PREFIX>
+static cudaError_t launch_tile_kernel(dim3 grid, const CUtensorMap &tk, const CUtensorMap &tv,
+                                      const KernelParams &p, cudaStream_t stream) {
+    static bool attr = false;
+    // the d = 64 tile is smaller; ask for the d = 128 footprint anyway so one
+    // CTA owns an SM (its 512 TMEM columns never wait on a neighbour)
+    if (!attr) {
+        cudaError_t e = cudaFuncSetAttribute(attn_tile_kernel<D, PREFIX>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             Layout<128>::kDynSmem);
+        if (e != cudaSuccess) return e;
+        attr = true;
+    }
+    attn_tile_kernel<D, PREFIX><<<grid, kThreads, Layout<128>::kDynSmem, stream>>>(tk, tv, p);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_prefill(const PrefillArgs &a, cudaStream_t stream, Tracer *tr) {
     const int g = a.Hq / a.Hkv;
@@ -386,31 +475,40 @@ cudaError_t launch_prefill(const PrefillArgs &a, cudaStream_t stream, Tracer *tr
     if (tiles <= 0 || a.R <= 0) return cudaSuccess;
     if (tiles > 65535) return cudaErrorInvalidConfiguration;
     dim3 grid((unsigned)(a.R * a.Hkv), (unsigned)tiles);
-    cudaError_t e;
     if (tr) tr->begin(kKernelPrefill, stream);
-    if (a.d == 128) {
-        static bool attr = false;
-        if (!attr) {
-            e = cudaFuncSetAttribute(prefill_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     Layout<128>::kDynSmem);
-            if (e != cudaSuccess) return e;
-            attr = true;
-        }
-        prefill_kernel<128><<<grid, kThreads, Layout<128>::kDynSmem, stream>>>(*a.tmap_k, *a.tmap_v, p);
-    } else {
-        static bool attr = false;
-        // the d = 64 tile is smaller; ask for the d = 128 footprint anyway so
-        // one CTA owns an SM (its 512 TMEM columns never wait on a neighbour)
-        if (!attr) {
-            e = cudaFuncSetAttribute(prefill_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     Layout<128>::kDynSmem);
-            if (e != cudaSuccess) return e;
-            attr = true;
-        }
-        prefill_kernel<64><<<grid, kThreads, Layout<128>::kDynSmem, stream>>>(*a.tmap_k, *a.tmap_v, p);
-    }
+    cudaError_t e = a.d == 128 ? launch_tile_kernel<128, false>(grid, *a.tmap_k, *a.tmap_v, p, stream)
+                               : launch_tile_kernel<64, false>(grid, *a.tmap_k, *a.tmap_v, p, stream);
     if (tr) tr->end(kKernelPrefill, stream);
-    return cudaGetLastError();
+    return e;
+}
+
+cudaError_t launch_decode_prefix(const DecodeLayout &L, const DecodeArgs &a,
+                                 int32_t num_blocks_pool, cudaStream_t stream, Tracer *tr) {
+    KernelParams p{};
+    p.q = static_cast<const uint16_t *>(a.q);
+    p.block_table = a.block_table;
+    p.max_blocks = a.max_blocks;
+    p.Hq = L.Hq; p.Hkv = L.Hkv; p.g = L.g; p.tpt = kRows / L.g;
+    p.num_blocks_pool = num_blocks_pool;
+    p.scale_log2 = a.scale_log2;
+    p.err = a.err;
+    p.group_start = a.group_start;
+    p.member_req = a.member_req;
+    p.group_blocks = a.group_blocks;
+    p.num_requests = L.R;
+    p.blocks_per_part = L.prefix_blocks_per_part;
+    p.parts_per_head = L.parts_per_head;
+    p.o_part = reinterpret_cast<float *>(static_cast<char *>(a.ws) + L.off_o);
+    p.ml_part = reinterpret_cast<float2 *>(static_cast<char *>(a.ws) + L.off_ml);
+    const int mtiles = (a.max_group_members + p.tpt - 1) / p.tpt;
+    if (mtiles <= 0 || L.prefix_parts <= 0) return cudaSuccess;
+    if (mtiles > 65535) return cudaErrorInvalidConfiguration;
+    dim3 grid((unsigned)(a.num_groups * L.Hkv), (unsigned)mtiles, (unsigned)L.prefix_parts);
+    if (tr) tr->begin(kKernelDecodePrefix, stream);
+    cudaError_t e = L.d == 128 ? launch_tile_kernel<128, true>(grid, *a.tmap_k, *a.tmap_v, p, stream)
+                               : launch_tile_kernel<64, true>(grid, *a.tmap_k, *a.tmap_v, p, stream);
+    if (tr) tr->end(kKernelDecodePrefix, stream);
+    return e;
 }
 
 }  // namespace pkv

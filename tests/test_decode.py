@@ -53,18 +53,38 @@ def compare(b, out, lse, reqs, threads=8):
     return e.max(), e.mean()
 
 
+@pytest.mark.parametrize("groups", [False, True])
 @pytest.mark.parametrize("name,scale", [
     ("tiny_decode", 1.0),
     ("l8b_decode", 0.25),     # 16 requests of full length
     ("qwen_mixed", 0.125),    # 32 decode requests over three prefixes, g = 7
     ("l70b_decode", 1 / 32),  # 16 requests, log-uniform suffixes, g = 8
 ])
-def test_decode_matches_oracle(name, scale):
+def test_decode_matches_oracle(name, scale, groups):
+    """groups=True: shared prefix blocks through the grouped prefix pass
+    (tcgen05) + private split pass + combine; False: split pass over all."""
     need_gpu()
     w = make_workload(name, scale_requests=scale)
     b = B.build_batch(w, poison=True)
-    out, lse = run_decode(b)
+    out, lse = run_decode(b, use_groups=groups)
     compare(b, out, lse, range(b.dec.start, b.dec.stop))
+    b.close()
+
+
+@pytest.mark.parametrize("name", ["l8b_decode", "qwen_mixed", "l70b_decode"])
+def test_decode_full_size_sampled_grouped(name):
+    """Full-size batch in the benchmark's launch configuration (grouped prefix
+    pass on): a sample of requests against the oracle, no NaN anywhere."""
+    need_gpu()
+    w = make_workload(name)
+    b = B.build_batch(w, poison=True)
+    out, lse = run_decode(b, use_groups=True)
+    assert torch.isfinite(out.float()).all()
+    ctx = w.context_lens[b.dec]
+    rng = np.random.default_rng(1)
+    picks = {0, len(ctx) - 1, int(np.argmin(ctx)), int(np.argmax(ctx))}
+    picks |= set(rng.choice(len(ctx), 4, replace=False).tolist())
+    compare(b, out, lse, [b.dec.start + i for i in sorted(picks)], threads=16)
     b.close()
 
 
@@ -86,7 +106,8 @@ def test_decode_full_size_sampled(name):
     b.close()
 
 
-def test_placement_invariance_bit_exact():
+@pytest.mark.parametrize("groups", [False, True])
+def test_placement_invariance_bit_exact(groups):
     """Different physical placements of the same logical cache give
     bit-identical outputs (the reduction order depends on positions only)."""
     need_gpu()
@@ -94,7 +115,7 @@ def test_placement_invariance_bit_exact():
     outs = []
     for seed in (0, 7, 123456789):
         b = B.build_batch(w, poison=True, placement_seed=seed)
-        o, l = run_decode(b)
+        o, l = run_decode(b, use_groups=groups)
         outs.append((o.cpu(), l.cpu()))
         b.close()
     for o, l in outs[1:]:
@@ -111,7 +132,27 @@ def test_shared_prefix_equals_private_copies():
     b2 = B.build_batch(w, poison=True, share_prefix=False)
     o2, l2 = run_decode(b2)
     assert torch.equal(o1, o2) and torch.equal(l1, l2)
+    # the grouped prefix pass reads the shared blocks once per group: same
+    # result up to summation order
+    o3, l3 = run_decode(b1, use_groups=True)
+    assert (o3.float() - o2.float()).abs().max().item() <= 2 * MAX_ABS / 2
+    assert (l3 - l2).abs().max().item() <= LSE_ABS
     b1.close(); b2.close()
+
+
+def test_grouped_members_need_not_be_contiguous():
+    """Group membership is a list: interleaved members of two groups."""
+    need_gpu()
+    R = 12
+    group = [i % 2 for i in range(R)]
+    w = make_workload("custom", custom=dict(Hq=16, Hkv=2, d=128, prefix_lens=[512, 1024],
+                                          group=group, cached=[(512 if g == 0 else 1024) + 40 + 7 * i
+                                                               for i, g in enumerate(group)],
+                                          new=[1] * R, decode=[True] * R))
+    b = B.build_batch(w, poison=True)
+    out, lse = run_decode(b, use_groups=True)
+    compare(b, out, lse, range(R))
+    b.close()
 
 
 def test_single_key_returns_value():
