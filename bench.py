@@ -417,6 +417,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--quick", action="store_true", help="headline workload only")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile", default=None, metavar="WORKLOAD",
+                    help="run only WORKLOAD's steps (for ncu captures); prints per-kernel times")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -433,6 +435,10 @@ def main():
     from paper_2605_11232_gb300 import pkv
     pkv.load()
     peaks = load_peaks()
+    if args.profile:
+        r = measure_workload(args.profile, args.steps, args.warmup)
+        print(json.dumps({"profile": args.profile, **summarize(r, peaks)}), flush=True)
+        return 0
     clocks = ClockSampler(local)
     clocks.start()
     time.sleep(0.3)

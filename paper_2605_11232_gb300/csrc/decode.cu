@@ -388,16 +388,28 @@ __global__ void __launch_bounds__(256) decode_combine_kernel(DecodeArgs a, Decod
     float acc[E];
 #pragma unroll
     for (int e = 0; e < E; ++e) acc[e] = 0.f;
-    for (int k = 0; k < total; ++k) {
-        const float wk = __shfl_sync(0xffffffffu, k < 32 ? w_a : w_b, k & 31);
-        const float *src = o_part + part_slot(k) * D + lane * E;
-        if constexpr (E == 4) {
-            const float4 v = *reinterpret_cast<const float4 *>(src);
-            acc[0] += wk * v.x; acc[1] += wk * v.y; acc[2] += wk * v.z; acc[3] += wk * v.w;
-        } else {
-            const float2 v = *reinterpret_cast<const float2 *>(src);
-            acc[0] += wk * v.x; acc[1] += wk * v.y;
+    // four parts per round: their loads are in flight together
+    for (int k0 = 0; k0 < total; k0 += 4) {
+        float v[4][E];
+        float wk[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int k = min(k0 + u, total - 1);
+            wk[u] = __shfl_sync(0xffffffffu, k < 32 ? w_a : w_b, k & 31);
+            if (k0 + u >= total) wk[u] = 0.f;
+            const float *src = o_part + part_slot(k) * D + lane * E;
+            if constexpr (E == 4) {
+                const float4 t = *reinterpret_cast<const float4 *>(src);
+                v[u][0] = t.x; v[u][1] = t.y; v[u][2] = t.z; v[u][3] = t.w;
+            } else {
+                const float2 t = *reinterpret_cast<const float2 *>(src);
+                v[u][0] = t.x; v[u][1] = t.y;
+            }
         }
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+            for (int e = 0; e < E; ++e) acc[e] += wk[u] * v[u][e];
     }
     uint16_t *out = static_cast<uint16_t *>(a.out) + item * D + lane * E;
     if constexpr (E == 4) {

@@ -40,6 +40,7 @@ constexpr int kKeys = 128;            // keys per tile (N of Q.K^T)
 constexpr uint32_t kTmemCols = 512;   // S0 [0,128) S1 [128,256) O [256, 256+D)
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr uint64_t kDrainLimitNs = 200000000ull;
+constexpr int kMaxItemBlocks = 2048;  // keys of one work item <= 32768
 
 template <int D>
 struct Layout {
@@ -54,7 +55,8 @@ struct Layout {
     static constexpr int kKFull = kBar + 0, kVFull = kBar + 16, kKvEmpty = kBar + 32;
     static constexpr int kSFull = kBar + 48, kPFull = kBar + 64, kOReady = kBar + 80;
     static constexpr int kDone = kBar + 88, kTmemSlot = kBar + 96, kAbort = kBar + 100;
-    static constexpr int kBytes = kBar + 128;
+    static constexpr int kBlkIds = kBar + 128;        // int32 [kMaxItemBlocks]
+    static constexpr int kBytes = kBlkIds + 4 * kMaxItemBlocks;
     static constexpr int kDynSmem = kBytes + 1024;    // room to align the base to 1 KiB
 };
 
@@ -162,6 +164,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         trow = p.block_table + (int64_t)r_first * p.max_blocks;
     }
+    if (nblk > kMaxItemBlocks) {
+        if (threadIdx.x == 0) latch_error(p.err, kDevBounds);
+        return;
+    }
     const int nkt = (kv_end + kKeys - 1) / kKeys;
     // global q row of tile row i (decode q is [R][Hq][D], prefill q is [T][Hq][D])
     auto q_row = [&](int i) -> int64_t {
@@ -196,18 +202,42 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_relinquish();
     }
     // Q tile -> shared memory, K-major with the 128-byte swizzle (16-byte
-    // chunk c of row i goes to chunk c ^ (i % 8) of its 128-byte row).
+    // chunk c of row i goes to chunk c ^ (i % 8) of its 128-byte row).  All
+    // loads are issued before the first store so their latencies overlap.
     {
         constexpr int kChunks = D / 8;
-        for (int idx = threadIdx.x; idx < kRows * kChunks; idx += kThreads) {
+        constexpr int kIters = (kRows * kChunks + kThreads - 1) / kThreads;
+        uint4 v[kIters];
+#pragma unroll
+        for (int k = 0; k < kIters; ++k) {
+            const int idx = threadIdx.x + k * kThreads;
             const int i = idx / kChunks, c = idx % kChunks;
-            uint4 v = make_uint4(0, 0, 0, 0);
-            if (i < rows_valid) v = ldg16(p.q + q_row(i) * D + c * 8);
-            const int half = c >> 3, cc = c & 7;
-            *reinterpret_cast<uint4 *>(smem + Ly::kQ + half * Ly::kHalfBytes + i * 128 +
-                                       ((cc ^ (i & 7)) << 4)) = v;
+            v[k] = make_uint4(0, 0, 0, 0);
+            if (idx < kRows * kChunks && i < rows_valid) v[k] = ldg16(p.q + q_row(i) * D + c * 8);
+        }
+#pragma unroll
+        for (int k = 0; k < kIters; ++k) {
+            const int idx = threadIdx.x + k * kThreads;
+            if (idx < kRows * kChunks) {
+                const int i = idx / kChunks, c = idx % kChunks;
+                const int half = c >> 3, cc = c & 7;
+                *reinterpret_cast<uint4 *>(smem + Ly::kQ + half * Ly::kHalfBytes + i * 128 +
+                                           ((cc ^ (i & 7)) << 4)) = v[k];
+            }
         }
         fence_proxy_async_smem();
+    }
+    // the item's physical block ids, checked once, for the producer
+    int32_t *blk_ids = reinterpret_cast<int32_t *>(smem + Ly::kBlkIds);
+    if (warp == 0) {
+        for (int b = lane; b < nblk; b += 32) {
+            int32_t id = __ldg(trow + blk_off + b);
+            if (id < 0 || id >= p.num_blocks_pool) {
+                latch_error(p.err, kDevBounds);
+                id = 0;
+            }
+            blk_ids[b] = id;
+        }
     }
     tc_fence_before();
     __syncthreads();
@@ -228,14 +258,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t kdst = sb + Ly::kK0 + s * Ly::kTile;
                 const uint32_t vdst = sb + Ly::kV0 + s * Ly::kTile;
                 int32_t phys[8];
-                for (int b = 0; b < nb; ++b) {
-                    int32_t id = __ldg(trow + blk_off + b0 + b);
-                    if (id < 0 || id >= p.num_blocks_pool) {
-                        latch_error(p.err, kDevBounds);
-                        id = 0;
-                    }
-                    phys[b] = id;
-                }
+                for (int b = 0; b < nb; ++b) phys[b] = blk_ids[b0 + b];
                 mbar_arrive_expect_tx(sb + Ly::kKFull + 8 * s, bytes);
                 for (int b = 0; b < nb; ++b)
                     for (int hf = 0; hf < Ly::kHalves; ++hf)
@@ -339,15 +362,23 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int kb = j * kKeys;
             const int lim = pos - kb;                 // keys with column index <= lim are visible
             float mx = -INFINITY;
+            if (__all_sync(0xffffffffu, lim >= kKeys - 1)) {
+                // every key of the tile is visible to every row of this warp
 #pragma unroll
-            for (int c = 0; c < 4; ++c)
+                for (int c = 0; c < 4; ++c)
 #pragma unroll
-                for (int e = 0; e < 32; ++e) {
-                    float v = __uint_as_float(sr[c][e]) * p.scale_log2;
-                    v = (c * 32 + e <= lim) ? v : -INFINITY;
-                    sr[c][e] = __float_as_uint(v);
-                    mx = fmaxf(mx, v);
-                }
+                    for (int e = 0; e < 32; ++e) mx = fmaxf(mx, __uint_as_float(sr[c][e]));
+            } else {
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) {
+                        const float v = (c * 32 + e <= lim) ? __uint_as_float(sr[c][e]) : -INFINITY;
+                        sr[c][e] = __float_as_uint(v);
+                        mx = fmaxf(mx, v);
+                    }
+            }
+            mx *= p.scale_log2;                       // scale > 0 commutes with max
             // conditional rescale: keep a stale max unless it grows by > 8 (x256)
             const float m_new = (mx > m + 8.0f) ? mx : m;
             const bool grow = (m_new != m) && (j > 0);
@@ -374,8 +405,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 uint32_t pk[16];
 #pragma unroll
                 for (int e = 0; e < 16; ++e) {
-                    const float p0 = fast_exp2(__uint_as_float(sr[c][2 * e]) - m);
-                    const float p1 = fast_exp2(__uint_as_float(sr[c][2 * e + 1]) - m);
+                    const float p0 = fast_exp2(fmaf(__uint_as_float(sr[c][2 * e]), p.scale_log2, -m));
+                    const float p1 = fast_exp2(fmaf(__uint_as_float(sr[c][2 * e + 1]), p.scale_log2, -m));
                     sum += p0 + p1;
                     pk[e] = pack_bf16x2(p0, p1);
                 }
