@@ -83,6 +83,27 @@ struct KernelParams {
     float2 *ml_part;            // [R*Hq*parts] (running max (base 2), sum)
 };
 
+// 2^x on the FMA pipe, to offload part of the exponentials from the
+// special-function unit (which alone would need as many cycles per score as
+// the two MMAs take).  x = n + f with n = round(x) found by adding
+// 1.5 * 2^23 (the sum's low mantissa bits are n), 2^f by a cubic fitted on
+// [-0.5, 0.5] (max relative error 7.5e-5; Lawson-weighted least squares on
+// Chebyshev nodes, see fit_exp2_poly.py), and n added into the exponent field.
+// x is clamped to -125 so the result stays a normal number; masked scores
+// (-inf) give exactly 0.
+__device__ __forceinline__ float poly_exp2(float x) {
+    const float xc = fmaxf(x, -125.0f);
+    const float t = xc + 12582912.0f;
+    const float n = t - 12582912.0f;
+    const float f = xc - n;
+    float p = fmaf(0.0551716648f, f, 0.2426111251f);
+    p = fmaf(p, f, 0.6932609677f);
+    p = fmaf(p, f, 0.9999280572f);
+    const uint32_t e = (uint32_t)(__float_as_int(t) - 0x4B400000) << 23;
+    const float r = __uint_as_float(__float_as_uint(p) + e);
+    return x < -125.0f ? 0.0f : r;
+}
+
 // TMEM address of the c-th 32-column chunk of the O accumulator in this
 // warp's lane quarter.
 __device__ __forceinline__ uint32_t o_addr(uint32_t tmem, uint32_t lane_off, int c) {
@@ -351,6 +372,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int pos = (!PREFIX && valid) ? q_pos0 + row / p.g : kv_end - 1;
         float m = -INFINITY, l = 0.f;
         bool ok = true;
+        // P.V completions (o_ready phases) consumed so far, in order
+        int o_seen = 0;
+        auto consume_o = [&](int upto) -> bool {
+            while (o_seen <= upto) {
+                if (!warp_wait(sb + Ly::kOReady, o_seen & 1, abort)) return false;
+                ++o_seen;
+            }
+            return true;
+        };
         for (int j = 0; j < nkt; ++j) {
             const int b = j & 1;
             if (!warp_wait(sb + Ly::kSFull + 8 * b, (j >> 1) & 1, abort)) { ok = false; break; }
@@ -383,19 +413,21 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float m_new = (mx > m + 8.0f) ? mx : m;
             const bool grow = (m_new != m) && (j > 0);
             float alpha = grow ? fast_exp2(m - m_new) : 1.0f;
-            if (j >= 1) {
-                if (!warp_wait(sb + Ly::kOReady, (j - 1) & 1, abort)) { ok = false; break; }
+            // P.V(j-2) finished before Q.K(j) (issued after it) did: consume
+            // its completion so this warp never lags the barrier by two phases
+            if (j >= 2 && !consume_o(j - 2)) { ok = false; break; }
+            if (__any_sync(0xffffffffu, grow)) {
+                // O must hold P.V(j-1) before it is rescaled
+                if (!consume_o(j - 1)) { ok = false; break; }
                 tc_fence_after();
-                if (__any_sync(0xffffffffu, grow)) {
 #pragma unroll
-                    for (int c = 0; c < D / 32; ++c) {
-                        uint32_t o[32];
-                        tmem_ld32(o_addr(tmem, lane_off, c), o);
-                        tmem_wait_ld();
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t o[32];
+                    tmem_ld32(o_addr(tmem, lane_off, c), o);
+                    tmem_wait_ld();
 #pragma unroll
-                        for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-                        tmem_st32(o_addr(tmem, lane_off, c), o);
-                    }
+                    for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+                    tmem_st32(o_addr(tmem, lane_off, c), o);
                 }
             }
             m = m_new;
@@ -405,8 +437,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 uint32_t pk[16];
 #pragma unroll
                 for (int e = 0; e < 16; ++e) {
-                    const float p0 = fast_exp2(fmaf(__uint_as_float(sr[c][2 * e]), p.scale_log2, -m));
-                    const float p1 = fast_exp2(fmaf(__uint_as_float(sr[c][2 * e + 1]), p.scale_log2, -m));
+                    const float x0 = fmaf(__uint_as_float(sr[c][2 * e]), p.scale_log2, -m);
+                    const float x1 = fmaf(__uint_as_float(sr[c][2 * e + 1]), p.scale_log2, -m);
+                    // one in four exponentials on the FMA pipe
+                    const float p0 = fast_exp2(x0);
+                    const float p1 = (e & 1) ? poly_exp2(x1) : fast_exp2(x1);
                     sum += p0 + p1;
                     pk[e] = pack_bf16x2(p0, p1);
                 }
@@ -417,7 +452,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_before();
             mbar_arrive(sb + Ly::kPFull + 8 * b);
         }
-        if (ok && warp_wait(sb + Ly::kOReady, (nkt - 1) & 1, abort)) {
+        if (ok && consume_o(nkt - 1)) {
             tc_fence_after();
             const int64_t orow = valid ? q_row(row) : 0;
             if constexpr (!PREFIX) {
