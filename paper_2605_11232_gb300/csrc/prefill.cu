@@ -51,10 +51,10 @@ struct Layout {
     static constexpr int kK0 = kQ + kTile;
     static constexpr int kV0 = kK0 + 2 * kTile;
     static constexpr int kBar = kV0 + 2 * kTile;
-    // barrier block: k_full[2] v_full[2] kv_empty[2] s_full[2] p_full[2] o_ready done
+    // barrier block: k_full[2] v_full[2] kv_empty[2] s_full[2] p_full[2] o_ready[2] done
     static constexpr int kKFull = kBar + 0, kVFull = kBar + 16, kKvEmpty = kBar + 32;
     static constexpr int kSFull = kBar + 48, kPFull = kBar + 64, kOReady = kBar + 80;
-    static constexpr int kDone = kBar + 88, kTmemSlot = kBar + 96, kAbort = kBar + 100;
+    static constexpr int kDone = kBar + 96, kTmemSlot = kBar + 104, kAbort = kBar + 108;
     static constexpr int kBlkIds = kBar + 128;        // int32 [kMaxItemBlocks]
     static constexpr int kBytes = kBlkIds + 4 * kMaxItemBlocks;
     static constexpr int kDynSmem = kBytes + 1024;    // room to align the base to 1 KiB
@@ -212,8 +212,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(sb + Ly::kKvEmpty + 8 * i, 1);
             mbar_init(sb + Ly::kSFull + 8 * i, 1);
             mbar_init(sb + Ly::kPFull + 8 * i, 128);
+            mbar_init(sb + Ly::kOReady + 8 * i, 1);
         }
-        mbar_init(sb + Ly::kOReady, 1);
         mbar_init(sb + Ly::kDone, 1);
         *abort = 0;
         fence_barrier_init();
@@ -334,7 +334,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mma_ts(o_col, tmem + s * 128 + kk * 8, bdesc, id_pv, (jj > 0 || kk > 0) ? 1u : 0u);
                 }
                 mma_commit(sb + Ly::kKvEmpty + 8 * s);
-                mma_commit(sb + Ly::kOReady);
+                mma_commit(sb + Ly::kOReady + 8 * (jj & 1));
             }
             __syncwarp();
             return true;
@@ -372,14 +372,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int pos = (!PREFIX && valid) ? q_pos0 + row / p.g : kv_end - 1;
         float m = -INFINITY, l = 0.f;
         bool ok = true;
-        // P.V completions (o_ready phases) consumed so far, in order
-        int o_seen = 0;
-        auto consume_o = [&](int upto) -> bool {
-            while (o_seen <= upto) {
-                if (!warp_wait(sb + Ly::kOReady, o_seen & 1, abort)) return false;
-                ++o_seen;
-            }
-            return true;
+        // P.V(k) completes o_ready[k & 1].  Waiting for P.V(k) is unambiguous
+        // when P.V(k - 2) is known complete, which holds wherever it is used
+        // below: Q.K(j) is issued after P.V(j - 2), and S(j) is in hand.
+        auto wait_pv = [&](int k) -> bool {
+            return warp_wait(sb + Ly::kOReady + 8 * (k & 1), (k >> 1) & 1, abort);
         };
         for (int j = 0; j < nkt; ++j) {
             const int b = j & 1;
@@ -413,12 +410,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float m_new = (mx > m + 8.0f) ? mx : m;
             const bool grow = (m_new != m) && (j > 0);
             float alpha = grow ? fast_exp2(m - m_new) : 1.0f;
-            // P.V(j-2) finished before Q.K(j) (issued after it) did: consume
-            // its completion so this warp never lags the barrier by two phases
-            if (j >= 2 && !consume_o(j - 2)) { ok = false; break; }
             if (__any_sync(0xffffffffu, grow)) {
                 // O must hold P.V(j-1) before it is rescaled
-                if (!consume_o(j - 1)) { ok = false; break; }
+                if (!wait_pv(j - 1)) { ok = false; break; }
                 tc_fence_after();
 #pragma unroll
                 for (int c = 0; c < D / 32; ++c) {
@@ -452,7 +446,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_before();
             mbar_arrive(sb + Ly::kPFull + 8 * b);
         }
-        if (ok && consume_o(nkt - 1)) {
+        if (ok && wait_pv(nkt - 1)) {
             tc_fence_after();
             const int64_t orow = valid ? q_row(row) : 0;
             if constexpr (!PREFIX) {
