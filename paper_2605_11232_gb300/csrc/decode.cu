@@ -435,8 +435,8 @@ DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_
         // Key splits of the prefix pass: one CTA per (group, kv head, member
         // tile, split), one CTA per SM.  Pick the split count that minimises
         // waves x (per-CTA set-up + key tiles per CTA), set-up ~ 2 key tiles.
-        const int tpt = 128 / L.g;
-        const int64_t tiles = (int64_t)num_groups * Hkv * ((max_group_members + tpt - 1) / tpt);
+        const int per_item = 2 * (128 / L.g);   // members per work item (two 128-row tiles)
+        const int64_t tiles = (int64_t)num_groups * Hkv * ((max_group_members + per_item - 1) / per_item);
         const int sms = num_sms > 0 ? num_sms : 148;
         const int key_tiles = (max_group_blocks + 7) / 8;
         int best = 1;
