@@ -10,7 +10,7 @@
 // the g q heads of a kv head sit next to each other (row = query * g + head),
 // so every K/V tile read serves all of them (GQA packing) and both tiles.
 //
-// Pipeline (one CTA per SM, 10 warps):
+// Pipeline (one CTA per SM, 12 warps = 3 warpgroups):
 //   warp 0     TMA producer: per 128-key tile, 8 paged blocks x head-dim
 //              halves of K and of V, each a 16-row x 128-byte box read
 //              through the block table, into a 2-stage ring (128-byte swizzle).
@@ -19,7 +19,8 @@
 //              so the tensor core runs one tile's MMAs while the other tile's
 //              softmax runs.  S = Q.K^T lands in TMEM; P.V reads P from TMEM
 //              and V from shared memory.
-//   warps 2-5  softmax of tile A, warps 6-9 of tile B: thread = row.  S row
+//   warps 2-3  idle (their warpgroup gives registers to the softmax ones)
+//   warps 4-7  softmax of tile A, warps 8-11 of tile B: thread = row.  S row
 //              from TMEM, causal mask, online max/sum in base 2 (tree
 //              reductions), P (bf16) written back over S in TMEM.  O is
 //              rescaled in TMEM only when the running max grows by more than
@@ -40,7 +41,13 @@ namespace {
 
 using namespace tc;
 
-constexpr int kThreads = 320;
+constexpr int kThreads = 384;
+// launch allocation 168 registers/thread (65536 / 384, rounded to 8); the
+// producer/MMA warpgroup drops to 56 and each softmax warpgroup rises to 224:
+// 56*128 + 2*224*128 = 168*384
+constexpr int kRegsLaunch = 168, kRegsControl = 56, kRegsSoftmax = 224;
+static_assert(kRegsControl * 128 + 2 * kRegsSoftmax * 128 == kRegsLaunch * kThreads,
+              "register split must add up to the launch allocation");
 constexpr int kRows = 128;            // M of one tile
 constexpr int kKeys = 128;            // keys per K/V tile (N of Q.K^T)
 constexpr uint32_t kTmemCols = 512;   // S_A [0,128) S_B [128,256) O_A [256,384) O_B [384,512)
@@ -128,7 +135,7 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
 //   the split's range of the group's prefix blocks (read through the first
 //   member's table row), all visible; writes unnormalised partials.
 template <int D, bool PREFIX>
-__global__ void __maxnreg__(200)   // 320 threads x 200 registers: one CTA per SM
+__global__ void __launch_bounds__(kThreads, 1)
     attn_tile_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
                      const KernelParams p) {
     using Ly = Layout<D>;
@@ -276,7 +283,9 @@ __global__ void __maxnreg__(200)   // 320 threads x 200 registers: one CTA per S
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp == 0) {
+    if (warp < 4) {
+      setmaxnreg_dec<kRegsControl>();
+      if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
             prefetch_tmap(&tmk);
@@ -391,9 +400,11 @@ __global__ void __maxnreg__(200)   // 320 threads x 200 registers: one CTA per S
         __syncwarp();
         int quiet = 0;
         mbar_wait(sb + Ly::kDone, 0, &quiet, kDrainLimitNs);
+      }
     } else {
+        setmaxnreg_inc<kRegsSoftmax>();
         // ------------------------------------------------------------ softmax
-        const int x = (warp - 2) >> 2;                // tile A (warps 2-5) or B (6-9)
+        const int x = (warp - 4) >> 2;                // tile A (warps 4-7) or B (8-11)
         const int quarter = warp & 3;                 // TMEM lanes this warp may touch
         const int row = quarter * 32 + lane;
         const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
