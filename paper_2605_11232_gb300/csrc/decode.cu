@@ -371,32 +371,22 @@ __global__ void __launch_bounds__(256) decode_combine_kernel(DecodeArgs a, Decod
     auto part_slot = [&](int k) {
         return slot0 + (k < n_pre ? k : lay.prefix_parts + (k - n_pre));
     };
-    // each lane holds up to two parts' (m, l)
-    float m_a = -INFINITY, l_a = 0.f, m_b = -INFINITY, l_b = 0.f;
-    if (lane < total) { float2 v = ml_part[part_slot(lane)]; m_a = v.x; l_a = v.y; }
-    if (lane + 32 < total) { float2 v = ml_part[part_slot(lane + 32)]; m_b = v.x; l_b = v.y; }
-    float mx = fmaxf(m_a, m_b);
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-    const float w_a = (lane < total) ? fast_exp2(m_a - mx) : 0.f;
-    const float w_b = (lane + 32 < total) ? fast_exp2(m_b - mx) : 0.f;
-    float den = w_a * l_a + w_b * l_b;
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) den += __shfl_xor_sync(0xffffffffu, den, off);
-    const float inv = 1.f / den;
     constexpr int E = D / 32;   // elements per lane
+    constexpr int kRound = 16;  // parts whose loads are in flight together
+    // each lane holds up to two parts' (m, l); issue those loads and the
+    // first round of partial-O loads before using either
+    float2 ml_a = make_float2(-INFINITY, 0.f), ml_b = make_float2(-INFINITY, 0.f);
+    if (lane < total) ml_a = ml_part[part_slot(lane)];
+    if (lane + 32 < total) ml_b = ml_part[part_slot(lane + 32)];
     float acc[E];
 #pragma unroll
     for (int e = 0; e < E; ++e) acc[e] = 0.f;
-    // four parts per round: their loads are in flight together
-    for (int k0 = 0; k0 < total; k0 += 4) {
-        float v[4][E];
-        float wk[4];
+    float mx = 0.f, w_a = 0.f, w_b = 0.f, den = 0.f;
+    for (int k0 = 0; k0 < total; k0 += kRound) {
+        float v[kRound][E];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
+        for (int u = 0; u < kRound; ++u) {
             const int k = min(k0 + u, total - 1);
-            wk[u] = __shfl_sync(0xffffffffu, k < 32 ? w_a : w_b, k & 31);
-            if (k0 + u >= total) wk[u] = 0.f;
             const float *src = o_part + part_slot(k) * D + lane * E;
             if constexpr (E == 4) {
                 const float4 t = *reinterpret_cast<const float4 *>(src);
@@ -406,11 +396,26 @@ __global__ void __launch_bounds__(256) decode_combine_kernel(DecodeArgs a, Decod
                 v[u][0] = t.x; v[u][1] = t.y;
             }
         }
+        if (k0 == 0) {
+            mx = fmaxf(ml_a.x, ml_b.x);
 #pragma unroll
-        for (int u = 0; u < 4; ++u)
+            for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+            w_a = (lane < total) ? fast_exp2(ml_a.x - mx) : 0.f;
+            w_b = (lane + 32 < total) ? fast_exp2(ml_b.x - mx) : 0.f;
+            den = w_a * ml_a.y + w_b * ml_b.y;
 #pragma unroll
-            for (int e = 0; e < E; ++e) acc[e] += wk[u] * v[u][e];
+            for (int off = 16; off > 0; off >>= 1) den += __shfl_xor_sync(0xffffffffu, den, off);
+        }
+#pragma unroll
+        for (int u = 0; u < kRound; ++u) {
+            const int k = k0 + u;
+            float wk = __shfl_sync(0xffffffffu, k < 32 ? w_a : w_b, k & 31);
+            if (k >= total) wk = 0.f;
+#pragma unroll
+            for (int e = 0; e < E; ++e) acc[e] += wk * v[u][e];
+        }
     }
+    const float inv = 1.f / den;
     uint16_t *out = static_cast<uint16_t *>(a.out) + item * D + lane * E;
     if constexpr (E == 4) {
         uint2 pk = make_uint2(pack_bf16x2(acc[0] * inv, acc[1] * inv),
