@@ -212,6 +212,29 @@ int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
                       float scale, const pkv_prefix_groups *groups, void *workspace,
                       size_t workspace_bytes, pkv_stream_t stream);
 
+/* ---- decode without a caller workspace ------------------------------------ */
+
+/* paged_attn_decode for callers that cannot allocate device memory when they
+ * decode (work recorded into a CUDA graph, inference plugins whose framework
+ * owns all device buffers, processes with a fixed up-front memory budget).
+ * The paper has no counterpart: this is a deployment convenience of the
+ * library.  Arguments and results are those of paged_attn_decode; the
+ * split-KV scratch comes from a 64 MiB static device array instead of a
+ * caller workspace, and the call allocates no device memory.
+ *  - Shapes whose workspace (paged_attn_decode_workspace_size) exceeds
+ *    64 MiB are refused with PKV_ERR_WORKSPACE.
+ *  - The first call on a device looks up the array's device address
+ *    (cudaGetSymbolAddress, with that device made current for the lookup);
+ *    make that first call before any stream capture.
+ *  - All calls share the one array: calls that may overlap on the GPU (other
+ *    streams, other threads, other pools on the same device) race on it and
+ *    must be serialised by the caller.
+ *  - Every GPU that loads the library holds the 64 MiB until process exit. */
+int paged_attn_decode_noalloc(pkv_pool_t pool, const void *q, void *out, float *lse,
+                              const int32_t *context_lens, const int32_t *block_table,
+                              int32_t max_blocks, int32_t num_requests, int32_t num_q_heads,
+                              float scale, const pkv_prefix_groups *groups, pkv_stream_t stream);
+
 /* ---- tracing -------------------------------------------------------------- */
 
 /* Per-kernel device time of the launches made while tracing was on. */

@@ -173,6 +173,14 @@ int build_tmaps(pkv_pool_t pool) {
 
 }  // namespace
 
+namespace pkv {
+// Record a failure message for pkv_last_error() from another translation unit.
+int set_last_error(int code, const char *msg) {
+    g_last_error = msg ? msg : "";
+    return code;
+}
+}  // namespace pkv
+
 extern "C" {
 
 const char *pkv_last_error(void) { return g_last_error.c_str(); }

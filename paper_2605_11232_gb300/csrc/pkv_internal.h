@@ -27,6 +27,9 @@ struct Tracer {
     virtual ~Tracer() {}
 };
 
+// Set the thread's pkv_last_error() message; returns code.
+int set_last_error(int code, const char *msg);
+
 // Device error word values (a kernel latches the first one with atomicCAS).
 enum : int {
     kDevOk = 0,

@@ -32,7 +32,7 @@ EXPORTS = [
     "kv_pool_create", "kv_pool_destroy", "kv_pool_alloc", "kv_pool_retain", "kv_pool_release",
     "kv_pool_refcount", "kv_pool_num_free", "kv_pool_alloc_sequence", "kv_slot_mapping",
     "kv_cache_write", "paged_attn_prefill", "paged_attn_decode_workspace_size",
-    "paged_attn_decode", "pkv_trace_enable", "pkv_trace_read", "pkv_check_device_errors",
+    "paged_attn_decode", "paged_attn_decode_noalloc", "pkv_trace_enable", "pkv_trace_read", "pkv_check_device_errors",
     "pkv_last_error",
 ]
 
@@ -94,6 +94,8 @@ def load(path: str | None = None):
         "paged_attn_decode": [V, V, V, V, V, V, i32, i32, i32, f32,
                               ctypes.POINTER(PrefixGroups), V, sz, V],
         "pkv_check_device_errors": [V, V, P],
+        "paged_attn_decode_noalloc": [V, V, V, V, V, V, i32, i32, i32, f32,
+                                      ctypes.POINTER(PrefixGroups), V],
         "pkv_trace_enable": [V, i32],
         "pkv_trace_read": [V, P, i32, P],
     }
@@ -239,6 +241,15 @@ def paged_attn_decode(pool, q, out, lse, context_lens, block_table, scale: float
         ctypes.byref(groups) if groups is not None else None, _dptr(workspace),
         int(workspace.numel() * workspace.element_size()) if workspace is not None else 0,
         _stream(stream)))
+
+
+def paged_attn_decode_noalloc(pool, q, out, lse, context_lens, block_table, scale: float,
+                              groups, stream=None):
+    """paged_attn_decode with the library's static scratch (no workspace)."""
+    _check(load().paged_attn_decode_noalloc(
+        pool, _dptr(q), _dptr(out), _dptr(lse), _dptr(context_lens), _dptr(block_table),
+        int(block_table.shape[1]), int(context_lens.shape[0]), int(q.shape[1]), float(scale),
+        ctypes.byref(groups) if groups is not None else None, _stream(stream)))
 
 
 def pkv_trace_enable(pool, enable: bool = True):
