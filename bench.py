@@ -382,31 +382,28 @@ METRIC = "prefix-cached paged-attn: prefill TFLOP/s & decode HBM GB/s, % of GB30
 
 
 def cpu_baseline(w_name, budget_s=12.0):
-    """The oracle as it stands on this host: decode requests of the headline
-    workload until about budget_s seconds of work, all host cores."""
+    """The oracle as it stands on this host: passes over the decode requests of
+    the headline workload until about budget_s seconds of work, all host cores."""
     import oracle
     from paper_2605_11232_gb300.workloads import make_workload
     cores = os.cpu_count() or 1
     w = make_workload(w_name)
+    per_pass_rows = sum(int(w.context_lens[r]) - w.prefix_len_of(r) for r in range(w.num_requests))
+    per_pass_rows += sum(w.prefix_lens[g] for g in {int(x) for x in w.group_of_req} if g >= 0)
+    per_pass = per_pass_rows * kv_row_bytes(w) + 2 * w.num_requests * w.num_q_heads * w.head_dim * 2
     t0 = time.perf_counter()
-    done, nbytes = 0, 0
-    groups = set()
-    rows = 0
-    for r in range(w.num_requests):
-        oracle.request_attention(w, r, threads=cores)
+    done = 0
+    while True:
+        for r in range(w.num_requests):
+            oracle.request_attention(w, r, threads=cores)
         done += 1
-        rows += int(w.context_lens[r]) - w.prefix_len_of(r)
-        if int(w.group_of_req[r]) >= 0:
-            groups.add(int(w.group_of_req[r]))
         if time.perf_counter() - t0 > budget_s:
             break
     dt = time.perf_counter() - t0
-    rows += sum(w.prefix_lens[g] for g in groups)
-    nbytes = rows * kv_row_bytes(w) + 2 * done * w.num_q_heads * w.head_dim * 2
-    return {"value": nbytes / dt / 1e9, "unit": "GB/s", "cores": cores, "kind": "oracle",
-            "sample": f"{done} of {w.num_requests} {w_name} decode requests (all q heads, full "
-                      f"context), fp64 C oracle, {cores} threads, {dt:.1f} s; bytes counted like the "
-                      "GPU metric (shared prefix once)"}
+    return {"value": done * per_pass / dt / 1e9, "unit": "GB/s", "cores": cores, "kind": "oracle",
+            "sample": f"{done} passes over all {w.num_requests} {w_name} decode requests (all q heads, "
+                      f"full context), fp64 C oracle, {cores} threads, {dt:.1f} s; bytes counted like "
+                      "the GPU metric (shared prefix once per pass)"}
 
 
 def main():
