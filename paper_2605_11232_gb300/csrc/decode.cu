@@ -228,7 +228,7 @@ template <int D, int NS>
 __global__ void __launch_bounds__(kThreads, 1) decode_split_kernel(DecodeArgs a, DecodeLayout lay,
                                                                   int32_t num_blocks_pool) {
     using Sm = SplitSmem<D>;
-    extern __shared__ __align__(1024) uint8_t dsmem[];
+    extern __shared__ __align__(128) uint8_t dsmem[];
     __shared__ int32_t s_max_n;
     const int32_t R = lay.R, Hkv = lay.Hkv, Hq = lay.Hq, g = lay.g;
     {
@@ -533,17 +533,29 @@ DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_
     return L;
 }
 
+// Largest dynamic shared memory a block of kernel k may request on this device.
+template <typename K>
+static size_t dyn_smem_limit(K k) {
+    int dev = 0, optin = 0;
+    cudaFuncAttributes fa{};
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
+        cudaFuncGetAttributes(&fa, k) != cudaSuccess)
+        return 0;
+    return optin > (int)fa.sharedSizeBytes ? (size_t)(optin - (int)fa.sharedSizeBytes) : 0;
+}
+
 template <int D, int NS>
 static cudaError_t launch_split(const DecodeLayout &L, const DecodeArgs &a, int num_sms,
                                 int32_t num_blocks_pool, cudaStream_t stream) {
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<D, NS>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    static size_t attr_bytes = 0;
     const size_t smem = SplitSmem<D>::bytes(NS, L.R);
+    if (smem > attr_bytes) {
+        cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<D, NS>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        attr_bytes = smem;
+    }
     decode_split_kernel<D, NS><<<num_sms, kThreads, smem, stream>>>(a, L, num_blocks_pool);
     return cudaGetLastError();
 }
@@ -557,7 +569,8 @@ static cudaError_t launch_decode_t(const DecodeLayout &L, const DecodeArgs &a, i
     }
     if (tr) tr->begin(kKernelDecodeSplit, stream);
     // three ring stages per warp while the request plan fits beside them
-    cudaError_t e = SplitSmem<D>::bytes(3, L.R) <= 227 * 1024
+    static const size_t limit3 = dyn_smem_limit(decode_split_kernel<D, 3>);
+    cudaError_t e = SplitSmem<D>::bytes(3, L.R) <= limit3
                         ? launch_split<D, 3>(L, a, num_sms, num_blocks_pool, stream)
                         : launch_split<D, 2>(L, a, num_sms, num_blocks_pool, stream);
     if (tr) tr->end(kKernelDecodeSplit, stream);
