@@ -14,11 +14,6 @@
 // segment it touches.  The combine kernel merges a head's partials with
 // log-sum-exp weights.
 //
-// Each warp streams its blocks through a private ring of NS shared-memory
-// stages (K tile + V tile of one block each), filled by TMA bulk copies and
-// tracked by one mbarrier per stage, so NS blocks per warp (NS x 8 KiB at
-// d = 128) are in flight while the warp computes.
-//
 // Inner loop (one 16-token block per step, per warp):
 //   S^T[16 keys x 8 heads] = K_blk[16 x d] . Q^T[d x 8]   (mma m16n8k16, A = K)
 //   online softmax per head column (shuffles across the 8 row groups)
@@ -34,7 +29,6 @@
 
 #include "pkv_device.cuh"
 #include "pkv_internal.h"
-#include "tc_ptx.cuh"
 
 namespace pkv {
 
@@ -59,22 +53,19 @@ struct BlockRegs {
     uint4 vb[D == 128 ? 4 : 1];   // V[4q+s][chunk 8+r] (d 64+8r..), d = 128 only
 };
 
-// Fragments of one block from its shared-memory stage (K tile then V tile,
-// each [16 keys][D] bf16 as in the pool).
 template <int D>
 __device__ __forceinline__ void load_block(BlockRegs<D> &b, const uint16_t *kt,
                                            const uint16_t *vt, int lr, int lq) {
     const int s0 = sigma(lr);
 #pragma unroll
     for (int j = 0; j < D / 32; ++j) {
-        b.ka[j] = *reinterpret_cast<const uint4 *>(kt + s0 * D + (4 * j + lq) * 8);
-        b.kb[j] = *reinterpret_cast<const uint4 *>(kt + (s0 + 2) * D + (4 * j + lq) * 8);
+        b.ka[j] = ldg_stream(kt + s0 * D + (4 * j + lq) * 8);
+        b.kb[j] = ldg_stream(kt + (s0 + 2) * D + (4 * j + lq) * 8);
     }
 #pragma unroll
     for (int s = 0; s < 4; ++s) {
-        b.va[s] = *reinterpret_cast<const uint4 *>(vt + (4 * lq + s) * D + lr * 8);
-        if constexpr (D == 128)
-            b.vb[s] = *reinterpret_cast<const uint4 *>(vt + (4 * lq + s) * D + (8 + lr) * 8);
+        b.va[s] = ldg_stream(vt + (4 * lq + s) * D + lr * 8);
+        if constexpr (D == 128) b.vb[s] = ldg_stream(vt + (4 * lq + s) * D + (8 + lr) * 8);
     }
 }
 
@@ -216,30 +207,11 @@ __device__ void build_plan(int32_t *P, int32_t R, const int32_t *__restrict__ co
 }
 
 template <int D>
-struct SplitSmem {
-    static constexpr int kTileBytes = 16 * D * 2;         // one (block, kv head) K or V tile
-    static constexpr int kStageBytes = 2 * kTileBytes;    // K then V
-    static constexpr size_t bytes(int ns, int R) {
-        return (size_t)kWarps * ns * kStageBytes + (size_t)kWarps * ns * 8 + (size_t)(R + 1) * 4;
-    }
-};
-
-template <int D, int NS>
 __global__ void __launch_bounds__(kThreads, 1) decode_split_kernel(DecodeArgs a, DecodeLayout lay,
                                                                   int32_t num_blocks_pool) {
-    using Sm = SplitSmem<D>;
-    extern __shared__ __align__(128) uint8_t dsmem[];
+    extern __shared__ int32_t P[];   // [R + 1]
     __shared__ int32_t s_max_n;
     const int32_t R = lay.R, Hkv = lay.Hkv, Hq = lay.Hq, g = lay.g;
-    {
-        // one mbarrier per ring stage, armed by the stage's copies
-        uint64_t *bars = reinterpret_cast<uint64_t *>(dsmem + (size_t)kWarps * NS * Sm::kStageBytes);
-        if (threadIdx.x < kWarps * NS) {
-            tc::mbar_init(tc::smem_u32(bars + threadIdx.x), 1);
-            tc::fence_barrier_init();
-        }
-    }
-    int32_t *P = reinterpret_cast<int32_t *>(dsmem + (size_t)kWarps * NS * (Sm::kStageBytes + 8));
     build_plan(P, R, a.context_lens, a.group_of_req, a.group_blocks, a.num_groups, a.max_blocks,
                &s_max_n, a.err);
     const int64_t W = (int64_t)Hkv * P[R];
@@ -252,11 +224,6 @@ __global__ void __launch_bounds__(kThreads, 1) decode_split_kernel(DecodeArgs a,
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int lr = lane >> 2, lq = lane & 3;
     const int64_t w = (int64_t)blockIdx.x * kWarps + warp;
-    uint8_t *ring = dsmem + (size_t)warp * NS * Sm::kStageBytes;
-    const uint32_t ring_s = tc::smem_u32(ring);
-    const uint32_t bar_s = tc::smem_u32(dsmem + (size_t)kWarps * NS * Sm::kStageBytes) + warp * NS * 8;
-    uint32_t n_issued = 0, n_used = 0;   // ring fills issued / consumed by this warp
-    bool ok = true;
     int64_t x = w * per;
     const int64_t x_end = min(x + per, W);
 
@@ -330,38 +297,16 @@ __global__ void __launch_bounds__(kThreads, 1) decode_split_kernel(DecodeArgs a,
             const int pos0 = (sh + b) * 16;
             return min(16, L - pos0);
         };
-        // fill the next ring stage with block b (whole warp calls; lane 0 copies)
-        auto issue = [&](int b) {
-            const uint16_t *kt = tile_of(b, kc);
-            const uint16_t *vt = tile_of(b, vc);
-            const uint32_t st_i = n_issued % NS;
-            if (lane == 0) {
-                const uint32_t bar = bar_s + st_i * 8;
-                const uint32_t dst = ring_s + st_i * Sm::kStageBytes;
-                tc::mbar_arrive_expect_tx(bar, Sm::kStageBytes);
-                tc::bulk_load(dst, kt, Sm::kTileBytes, bar);
-                tc::bulk_load(dst + Sm::kTileBytes, vt, Sm::kTileBytes, bar);
-            }
-            ++n_issued;
-        };
-        for (int k = 0; k < NS && b_lo + k < b_hi; ++k) issue(b_lo + k);
-        for (int b = b_lo; b < b_hi; ++b) {
-            const uint32_t st_i = n_used % NS;
-            int quiet = 0;
-            if (!__all_sync(0xffffffffu, tc::mbar_wait(bar_s + st_i * 8, (n_used / NS) & 1, &quiet,
-                                                       2000000000ull))) {
-                ok = false;
-                break;
-            }
-            const uint16_t *kt = reinterpret_cast<const uint16_t *>(ring + st_i * Sm::kStageBytes);
-            BlockRegs<D> br;
-            load_block<D>(br, kt, kt + Sm::kTileBytes / 2, lr, lq);
-            attend_block<D>(st, br, qf, lr, lq, valid_of(b), a.scale_log2);
-            ++n_used;
-            __syncwarp();   // every lane is done with the stage before it is refilled
-            if (b + NS < b_hi) issue(b + NS);
+
+        BlockRegs<D> b0, b1;
+        load_block<D>(b0, tile_of(b_lo, kc), tile_of(b_lo, vc), lr, lq);
+        for (int b = b_lo; b < b_hi; b += 2) {
+            if (b + 1 < b_hi) load_block<D>(b1, tile_of(b + 1, kc), tile_of(b + 1, vc), lr, lq);
+            attend_block<D>(st, b0, qf, lr, lq, valid_of(b), a.scale_log2);
+            if (b + 1 >= b_hi) break;
+            if (b + 2 < b_hi) load_block<D>(b0, tile_of(b + 2, kc), tile_of(b + 2, vc), lr, lq);
+            attend_block<D>(st, b1, qf, lr, lq, valid_of(b + 1), a.scale_log2);
         }
-        if (!ok) break;
 
         // row-group reduction of the thread-partial sums
 #pragma unroll
@@ -394,15 +339,6 @@ __global__ void __launch_bounds__(kThreads, 1) decode_split_kernel(DecodeArgs a,
             nparts[(int64_t)r * Hkv + h] = (int32_t)((seg_off + n - 1) / per - seg_off / per + 1);
         }
         x = piece_end;
-    }
-    if (!ok) {
-        // a stage wait ran out: report it and let this warp's copies land
-        // (bounded) before the CTA's shared memory is released
-        if (lane == 0) latch_error(a.err, kDevTimeout);
-        for (; n_used < n_issued; ++n_used) {
-            int quiet = 0;
-            tc::mbar_wait(bar_s + (n_used % NS) * 8, (n_used / NS) & 1, &quiet, 200000000ull);
-        }
     }
 }
 
@@ -533,33 +469,6 @@ DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_
     return L;
 }
 
-// Largest dynamic shared memory a block of kernel k may request on this device.
-template <typename K>
-static size_t dyn_smem_limit(K k) {
-    int dev = 0, optin = 0;
-    cudaFuncAttributes fa{};
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
-        cudaFuncGetAttributes(&fa, k) != cudaSuccess)
-        return 0;
-    return optin > (int)fa.sharedSizeBytes ? (size_t)(optin - (int)fa.sharedSizeBytes) : 0;
-}
-
-template <int D, int NS>
-static cudaError_t launch_split(const DecodeLayout &L, const DecodeArgs &a, int num_sms,
-                                int32_t num_blocks_pool, cudaStream_t stream) {
-    static size_t attr_bytes = 0;
-    const size_t smem = SplitSmem<D>::bytes(NS, L.R);
-    if (smem > attr_bytes) {
-        cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<D, NS>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        attr_bytes = smem;
-    }
-    decode_split_kernel<D, NS><<<num_sms, kThreads, smem, stream>>>(a, L, num_blocks_pool);
-    return cudaGetLastError();
-}
-
 template <int D>
 static cudaError_t launch_decode_t(const DecodeLayout &L, const DecodeArgs &a, int num_sms,
                                    int32_t num_blocks_pool, cudaStream_t stream, Tracer *tr) {
@@ -567,13 +476,18 @@ static cudaError_t launch_decode_t(const DecodeLayout &L, const DecodeArgs &a, i
         cudaError_t e = launch_decode_prefix(L, a, num_blocks_pool, stream, tr);
         if (e != cudaSuccess) return e;
     }
+    const size_t smem = (size_t)(L.R + 1) * sizeof(int32_t);
+    static size_t attr_bytes = 0;
+    if (smem > 48 * 1024 && smem > attr_bytes) {
+        cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<D>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        attr_bytes = smem;
+    }
     if (tr) tr->begin(kKernelDecodeSplit, stream);
-    // three ring stages per warp while the request plan fits beside them
-    static const size_t limit3 = dyn_smem_limit(decode_split_kernel<D, 3>);
-    cudaError_t e = SplitSmem<D>::bytes(3, L.R) <= limit3
-                        ? launch_split<D, 3>(L, a, num_sms, num_blocks_pool, stream)
-                        : launch_split<D, 2>(L, a, num_sms, num_blocks_pool, stream);
+    decode_split_kernel<D><<<num_sms, kThreads, smem, stream>>>(a, L, num_blocks_pool);
     if (tr) tr->end(kKernelDecodeSplit, stream);
+    cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const int64_t items = (int64_t)L.R * L.Hq;
     const int64_t grid = (items + 7) / 8;

@@ -488,44 +488,73 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (ok && warp_wait(sb + Ly::kODone + 8 * x, 0, abort)) {
             tc_fence_after();
-            const int64_t orow = valid ? q_row(qi, row % p.g) : 0;
+            // Epilogue through shared memory: every MMA reading Q_X has
+            // finished, so this tile's Q buffer holds the rows while they are
+            // turned from one-row-per-thread into whole-row 16-byte stores.
+            // Staged rows are RB = 2*D bytes (128 rows fill the Q tile); 16-byte
+            // chunk c of row i sits at chunk c ^ (i % CPR), so both the
+            // per-row writes and the per-chunk reads avoid bank conflicts.
+            uint8_t *stage = smem + Ly::kQ + x * Ly::kTile;
+            constexpr int RB = 2 * D, CPR = RB / 16, RPI = 32 / CPR;
+            static_assert(kRows * RB == Ly::kTile, "staging rows must fill the Q tile");
+            auto row_chunk = [&](int i, int c) -> uint4 * {
+                return reinterpret_cast<uint4 *>(stage + i * RB + ((c ^ (i & (CPR - 1))) << 4));
+            };
+            // drain the staged rows of this warp: lane -> (row, chunk)
+            auto drain = [&](auto &&dst_of) {
+                __syncwarp();
+#pragma unroll
+                for (int it = 0; it < 32 / RPI; ++it) {
+                    const int i = quarter * 32 + it * RPI + lane / CPR, c = lane % CPR;
+                    const uint4 v = *row_chunk(i, c);
+                    if (i < rows_x) *dst_of(i, c) = v;
+                }
+                __syncwarp();
+            };
             if constexpr (!PREFIX) {
                 const float inv = 1.0f / l;
+                // bf16 rows of D values: D * 2 bytes <= RB
 #pragma unroll
                 for (int c = 0; c < D / 32; ++c) {
                     uint32_t o[32];
                     tmem_ld32(o_addr + c * 32, o);
                     tmem_wait_ld();
-                    if (valid) {
-                        uint4 *dst = reinterpret_cast<uint4 *>(p.out + orow * D + c * 32);
 #pragma unroll
-                        for (int v = 0; v < 4; ++v) {
-                            uint4 w;
-                            w.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv, __uint_as_float(o[8 * v + 1]) * inv);
-                            w.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv, __uint_as_float(o[8 * v + 3]) * inv);
-                            w.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv, __uint_as_float(o[8 * v + 5]) * inv);
-                            w.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv, __uint_as_float(o[8 * v + 7]) * inv);
-                            dst[v] = w;
-                        }
+                    for (int v = 0; v < 4; ++v) {
+                        uint4 w;
+                        w.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv, __uint_as_float(o[8 * v + 1]) * inv);
+                        w.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv, __uint_as_float(o[8 * v + 3]) * inv);
+                        w.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv, __uint_as_float(o[8 * v + 5]) * inv);
+                        w.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv, __uint_as_float(o[8 * v + 7]) * inv);
+                        *row_chunk(row, 4 * c + v) = w;
                     }
                 }
-                if (valid && p.lse) p.lse[orow] = (m + __log2f(l)) * 0.69314718055994530942f;
+                drain([&](int i, int c) {
+                    const int64_t orow = q_row(x * p.tpt + i / p.g, i % p.g);
+                    return reinterpret_cast<uint4 *>(p.out + orow * D) + c;
+                });
+                if (valid && p.lse)
+                    p.lse[q_row(qi, row % p.g)] = (m + __log2f(l)) * 0.69314718055994530942f;
             } else {
-                // unnormalised partial of key split blockIdx.z, merged by the combine
-                const int64_t slot = orow * p.parts_per_head + blockIdx.z;
+                // unnormalised fp32 partial of key split blockIdx.z, merged by
+                // the combine; staged D/2 columns (RB bytes) at a time
 #pragma unroll
-                for (int c = 0; c < D / 32; ++c) {
-                    uint32_t o[32];
-                    tmem_ld32(o_addr + c * 32, o);
-                    tmem_wait_ld();
-                    if (valid) {
-                        uint4 *dst = reinterpret_cast<uint4 *>(p.o_part + slot * D + c * 32);
+                for (int hc = 0; hc < 2; ++hc) {
+#pragma unroll
+                    for (int cc = 0; cc < D / 64; ++cc) {
+                        uint32_t o[32];
+                        tmem_ld32(o_addr + hc * (D / 2) + cc * 32, o);
+                        tmem_wait_ld();
 #pragma unroll
                         for (int v = 0; v < 8; ++v)
-                            dst[v] = make_uint4(o[4 * v], o[4 * v + 1], o[4 * v + 2], o[4 * v + 3]);
+                            *row_chunk(row, 8 * cc + v) = make_uint4(o[4 * v], o[4 * v + 1], o[4 * v + 2], o[4 * v + 3]);
                     }
+                    drain([&](int i, int c) {
+                        const int64_t slot = q_row(x * p.tpt + i / p.g, i % p.g) * p.parts_per_head + blockIdx.z;
+                        return reinterpret_cast<uint4 *>(p.o_part + slot * D + hc * (D / 2)) + c;
+                    });
                 }
-                if (valid) p.ml_part[slot] = make_float2(m, l);
+                if (valid) p.ml_part[q_row(qi, row % p.g) * p.parts_per_head + blockIdx.z] = make_float2(m, l);
             }
         }
     }
