@@ -65,11 +65,14 @@ struct Layout {
     static constexpr int kV0 = kK0 + 2 * kTile;
     static constexpr int kBar = kV0 + 2 * kTile;
     // barriers: k_full[2] v_full[2] kv_empty[2] s_full[A,B] p_full[A,B] o_done[A,B] done
+    // turn[A,B] (the two softmax warpgroups take turns)
     static constexpr int kKFull = kBar + 0, kVFull = kBar + 16, kKvEmpty = kBar + 32;
     static constexpr int kSFull = kBar + 48, kPFull = kBar + 64, kODone = kBar + 80;
-    static constexpr int kDone = kBar + 96, kTmemSlot = kBar + 104, kAbort = kBar + 108;
+    static constexpr int kDone = kBar + 96, kTurn = kBar + 104;
+    static constexpr int kTmemSlot = kBar + 120, kAbort = kBar + 124;
     static constexpr int kBlkIds = kBar + 128;        // int32 [kMaxItemBlocks]
-    static constexpr int kBytes = kBlkIds + 4 * kMaxItemBlocks;
+    static constexpr int kRowIdx = kBlkIds + 4 * kMaxItemBlocks;   // int64 [2 * kRows]
+    static constexpr int kBytes = kRowIdx + 8 * 2 * kRows;
     static constexpr int kDynSmem = kBytes + 1024;    // room to align the base to 1 KiB
 };
 
@@ -96,25 +99,26 @@ struct KernelParams {
     float2 *ml_part;            // [R*Hq*parts] (running max (base 2), sum)
 };
 
-// 2^x on the FMA pipe, to offload part of the exponentials from the
-// special-function unit (which alone would need as many cycles per score as
-// the two MMAs take).  x = n + f with n = round(x) found by adding
-// 1.5 * 2^23 (the sum's low mantissa bits are n), 2^f by a cubic fitted on
-// [-0.5, 0.5] (max relative error 7.5e-5; Lawson-weighted least squares on
-// Chebyshev nodes, see fit_exp2_poly.py), and n added into the exponent field.
-// x is clamped to -125 so the result stays a normal number; masked scores
-// (-inf) give exactly 0.
-__device__ __forceinline__ float poly_exp2(float x) {
-    const float xc = fmaxf(x, -125.0f);
-    const float t = xc + 12582912.0f;
-    const float n = t - 12582912.0f;
-    const float f = xc - n;
-    float p = fmaf(0.0551716648f, f, 0.2426111251f);
-    p = fmaf(p, f, 0.6932609677f);
-    p = fmaf(p, f, 0.9999280572f);
-    const uint32_t e = (uint32_t)(__float_as_int(t) - 0x4B400000) << 23;
-    const float r = __uint_as_float(__float_as_uint(p) + e);
-    return x < -125.0f ? 0.0f : r;
+// 2^x for two values on the FMA pipe (packed fp32), to offload half of the
+// exponentials from the special-function unit, which alone would need as many
+// cycles per score as the two MMAs take.  x = n + f with n = round(x) found
+// by adding 1.5 * 2^23 (the sum's low mantissa bits hold n), 2^f by a cubic
+// fitted on [-0.5, 0.5] (max relative error 7.5e-5; Lawson-weighted least
+// squares on Chebyshev nodes, see fit_exp2_poly.py), and n added into the
+// exponent field: bits(p) + (n << 23) is one multiply-add on bits(t), since
+// 0x4B400000 << 23 wraps to 0.  x is clamped to -125 so the result stays a
+// normal number; inputs must be finite (masked tiles use the SFU instead).
+__device__ __forceinline__ float2 poly_exp2_x2(float2 x) {
+    const float2 xc = make_float2(fmaxf(x.x, -125.0f), fmaxf(x.y, -125.0f));
+    const float2 t = fadd2(xc, make_float2(12582912.0f, 12582912.0f));
+    const float2 n = fadd2(t, make_float2(-12582912.0f, -12582912.0f));
+    const float2 f = fadd2(xc, make_float2(-n.x, -n.y));
+    float2 p = ffma2(make_float2(0.0551716648f, 0.0551716648f), f,
+                     make_float2(0.2426111251f, 0.2426111251f));
+    p = ffma2(p, f, make_float2(0.6932609677f, 0.6932609677f));
+    p = ffma2(p, f, make_float2(0.9999280572f, 0.9999280572f));
+    return make_float2(__uint_as_float(__float_as_uint(t.x) * 0x800000u + __float_as_uint(p.x)),
+                       __uint_as_float(__float_as_uint(t.y) * 0x800000u + __float_as_uint(p.y)));
 }
 
 __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile int *abort) {
@@ -223,6 +227,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(sb + Ly::kSFull + 8 * i, 1);
             mbar_init(sb + Ly::kPFull + 8 * i, 128);
             mbar_init(sb + Ly::kODone + 8 * i, 1);
+            mbar_init(sb + Ly::kTurn + 8 * i, 128);
         }
         mbar_init(sb + Ly::kDone, 1);
         *abort = 0;
@@ -232,9 +237,27 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_alloc(smem_u32(tmem_slot), kTmemCols);
         tmem_relinquish();
     }
+    // global q row of every tile row (-1: no query), looked up once; the Q
+    // loads and the epilogue stores use this table
+    int64_t *row_idx = reinterpret_cast<int64_t *>(smem + Ly::kRowIdx);
+    if (threadIdx.x < 2 * kRows) {
+        const int x = threadIdx.x >> 7, i = threadIdx.x & 127;
+        row_idx[threadIdx.x] = i < (x ? rows_b : rows_a) ? q_row(x * p.tpt + i / p.g, i % p.g) : -1;
+    }
+    // the item's physical block ids, checked once, for the producer
+    int32_t *blk_ids = reinterpret_cast<int32_t *>(smem + Ly::kBlkIds);
+    for (int b = threadIdx.x - 2 * kRows; b >= 0 && b < nblk; b += kThreads - 2 * kRows) {
+        int32_t id = __ldg(trow + blk_off + b);
+        if (id < 0 || id >= p.num_blocks_pool) {
+            latch_error(p.err, kDevBounds);
+            id = 0;
+        }
+        blk_ids[b] = id;
+    }
+    __syncthreads();
     // Q tiles -> shared memory, K-major with the 128-byte swizzle (16-byte
     // chunk c of row i goes to chunk c ^ (i % 8) of its 128-byte row).  All
-    // loads are issued before the first store so their latencies overlap.
+    // loads of a round are issued before its first store.
     {
         constexpr int kChunks = D / 8;
         constexpr int kTotal = 2 * kRows * kChunks;
@@ -247,10 +270,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int k = 0; k < kHalfIters; ++k) {
                 const int idx = threadIdx.x + (round * kHalfIters + k) * kThreads;
                 const int row = idx / kChunks, c = idx % kChunks;
-                const int x = row >> 7, i = row & 127;
                 v[k] = make_uint4(0, 0, 0, 0);
-                if (idx < kTotal && i < (x ? rows_b : rows_a))
-                    v[k] = ldg16(p.q + q_row(x * p.tpt + i / p.g, i % p.g) * D + c * 8);
+                if (idx < kTotal) {
+                    const int64_t qr = row_idx[row];
+                    if (qr >= 0) v[k] = ldg16(p.q + qr * D + c * 8);
+                }
             }
 #pragma unroll
             for (int k = 0; k < kHalfIters; ++k) {
@@ -265,18 +289,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
         fence_proxy_async_smem();
-    }
-    // the item's physical block ids, checked once, for the producer
-    int32_t *blk_ids = reinterpret_cast<int32_t *>(smem + Ly::kBlkIds);
-    if (warp == 0) {
-        for (int b = lane; b < nblk; b += 32) {
-            int32_t id = __ldg(trow + blk_off + b);
-            if (id < 0 || id >= p.num_blocks_pool) {
-                latch_error(p.err, kDevBounds);
-                id = 0;
-            }
-            blk_ids[b] = id;
-        }
     }
     tc_fence_before();
     __syncthreads();
@@ -420,21 +432,32 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool ok = active;
         for (int j = 0; j < nkt && ok; ++j) {
             if (!warp_wait(sb + Ly::kSFull + 8 * x, j & 1, abort)) { ok = false; break; }
+            // take turns with the other tile's warpgroup, so that one group's
+            // softmax overlaps the other group's MMAs instead of competing for
+            // the same issue slots and SFU (turn[A] is completed by B after
+            // its tile j-1, turn[B] by A after its tile j)
+            if (has_b && (x == 1 || j >= 1) &&
+                !warp_wait(sb + Ly::kTurn + 8 * x, (x ? j : j - 1) & 1, abort)) {
+                ok = false;
+                break;
+            }
             tc_fence_after();
             uint32_t sr[4][32];
 #pragma unroll
             for (int c = 0; c < 4; ++c) tmem_ld32(s_addr + c * 32, sr[c]);
             tmem_wait_ld();
             const int lim = pos - j * kKeys;          // keys with column index <= lim are visible
+            const bool all_visible = __all_sync(0xffffffffu, lim >= kKeys - 1);
             float mx8[8];
 #pragma unroll
             for (int t = 0; t < 8; ++t) mx8[t] = -INFINITY;
-            if (__all_sync(0xffffffffu, lim >= kKeys - 1)) {
-                // every key of the tile is visible to every row of this warp
+            if (all_visible) {
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
 #pragma unroll
-                    for (int e = 0; e < 32; ++e) mx8[e & 7] = fmaxf(mx8[e & 7], __uint_as_float(sr[c][e]));
+                    for (int e = 0; e < 32; e += 2)
+                        mx8[(e >> 1) & 7] = fmax3(mx8[(e >> 1) & 7], __uint_as_float(sr[c][e]),
+                                                  __uint_as_float(sr[c][e + 1]));
             } else {
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
@@ -445,8 +468,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         mx8[e & 7] = fmaxf(mx8[e & 7], v);
                     }
             }
-            const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                                   fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]))) *
+            const float mx = fmaxf(fmax3(mx8[0], mx8[1], mx8[2]),
+                                   fmax3(fmax3(mx8[3], mx8[4], mx8[5]), mx8[6], mx8[7])) *
                              p.scale_log2;            // scale > 0 commutes with max
             // conditional rescale: keep a stale max unless it grows by > 8 (x256)
             const float m_new = (mx > m + 8.0f) ? mx : m;
@@ -465,26 +488,48 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
             m = m_new;
-            float sum4[4] = {0.f, 0.f, 0.f, 0.f};
+            const float2 sc2 = make_float2(p.scale_log2, p.scale_log2);
+            const float2 nm2 = make_float2(-m, -m);
+            float2 sum2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+            if (all_visible) {
+                // half of the exponentials on the FMA pipe (packed cubic), half on the SFU
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                uint32_t pk[16];
+                for (int c = 0; c < 4; ++c) {
+                    uint32_t pk[16];
 #pragma unroll
-                for (int e = 0; e < 16; ++e) {
-                    const float x0 = fmaf(__uint_as_float(sr[c][2 * e]), p.scale_log2, -m);
-                    const float x1 = fmaf(__uint_as_float(sr[c][2 * e + 1]), p.scale_log2, -m);
-                    // one in four exponentials on the FMA pipe
-                    const float p0 = fast_exp2(x0);
-                    const float p1 = (e & 1) ? poly_exp2(x1) : fast_exp2(x1);
-                    sum4[e & 3] += p0 + p1;
-                    pk[e] = pack_bf16x2(p0, p1);
+                    for (int e = 0; e < 16; ++e) {
+                        const float2 xv = ffma2(make_float2(__uint_as_float(sr[c][2 * e]),
+                                                            __uint_as_float(sr[c][2 * e + 1])), sc2, nm2);
+                        const float2 pp = (e & 1) ? poly_exp2_x2(xv)
+                                                  : make_float2(fast_exp2(xv.x), fast_exp2(xv.y));
+                        sum2[e & 1] = fadd2(sum2[e & 1], pp);
+                        pk[e] = pack_bf16x2(pp.x, pp.y);
+                    }
+                    tmem_st16(s_addr + c * 16, pk);
                 }
-                tmem_st16(s_addr + c * 16, pk);
+            } else {
+                // masked tile: SFU only, so masked scores (-inf) give exactly 0
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    uint32_t pk[16];
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) {
+                        const float2 xv = ffma2(make_float2(__uint_as_float(sr[c][2 * e]),
+                                                            __uint_as_float(sr[c][2 * e + 1])), sc2, nm2);
+                        const float2 pp = make_float2(fast_exp2(xv.x), fast_exp2(xv.y));
+                        sum2[e & 1] = fadd2(sum2[e & 1], pp);
+                        pk[e] = pack_bf16x2(pp.x, pp.y);
+                    }
+                    tmem_st16(s_addr + c * 16, pk);
+                }
             }
-            l = l * alpha + ((sum4[0] + sum4[1]) + (sum4[2] + sum4[3]));
+            const float2 s2 = fadd2(sum2[0], sum2[1]);
+            l = l * alpha + (s2.x + s2.y);
             tmem_wait_st();
             tc_fence_before();
             mbar_arrive(sb + Ly::kPFull + 8 * x);
+            // hand the turn to the other warpgroup
+            if (has_b && (x == 0 || j + 1 < nkt)) mbar_arrive(sb + Ly::kTurn + 8 * (x ^ 1));
         }
         if (ok && warp_wait(sb + Ly::kODone + 8 * x, 0, abort)) {
             tc_fence_after();
@@ -530,11 +575,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
                 drain([&](int i, int c) {
-                    const int64_t orow = q_row(x * p.tpt + i / p.g, i % p.g);
-                    return reinterpret_cast<uint4 *>(p.out + orow * D) + c;
+                    return reinterpret_cast<uint4 *>(p.out + row_idx[x * kRows + i] * D) + c;
                 });
-                if (valid && p.lse)
-                    p.lse[q_row(qi, row % p.g)] = (m + __log2f(l)) * 0.69314718055994530942f;
+                if (valid && p.lse) p.lse[row_idx[x * kRows + row]] = (m + __log2f(l)) * 0.69314718055994530942f;
             } else {
                 // unnormalised fp32 partial of key split blockIdx.z, merged by
                 // the combine; staged D/2 columns (RB bytes) at a time
@@ -550,11 +593,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                             *row_chunk(row, 8 * cc + v) = make_uint4(o[4 * v], o[4 * v + 1], o[4 * v + 2], o[4 * v + 3]);
                     }
                     drain([&](int i, int c) {
-                        const int64_t slot = q_row(x * p.tpt + i / p.g, i % p.g) * p.parts_per_head + blockIdx.z;
+                        const int64_t slot = row_idx[x * kRows + i] * p.parts_per_head + blockIdx.z;
                         return reinterpret_cast<uint4 *>(p.o_part + slot * D + hc * (D / 2)) + c;
                     });
                 }
-                if (valid) p.ml_part[q_row(qi, row % p.g) * p.parts_per_head + blockIdx.z] = make_float2(m, l);
+                if (valid) p.ml_part[row_idx[x * kRows + row] * p.parts_per_head + blockIdx.z] = make_float2(m, l);
             }
         }
     }
