@@ -64,13 +64,13 @@ struct Layout {
     static constexpr int kK0 = kQ + 2 * kTile;
     static constexpr int kV0 = kK0 + 2 * kTile;
     static constexpr int kBar = kV0 + 2 * kTile;
-    // barriers: k_full[2] v_full[2] kv_empty[2] s_full[A,B] p_full[A,B] o_done[A,B] done
-    // turn[A,B] (the two softmax warpgroups take turns)
-    static constexpr int kKFull = kBar + 0, kVFull = kBar + 16, kKvEmpty = kBar + 32;
-    static constexpr int kSFull = kBar + 48, kPFull = kBar + 64, kODone = kBar + 80;
-    static constexpr int kDone = kBar + 96, kTurn = kBar + 104;
-    static constexpr int kTmemSlot = kBar + 120, kAbort = kBar + 124;
-    static constexpr int kBlkIds = kBar + 128;        // int32 [kMaxItemBlocks]
+    // barriers: k_full[2] v_full[2] k_empty[2] v_empty[2] s_full[A,B] p_full[A,B]
+    // o_done[A,B] turn[A,B] (the softmax warpgroups take turns) done
+    static constexpr int kKFull = kBar + 0, kVFull = kBar + 16, kKEmpty = kBar + 32;
+    static constexpr int kVEmpty = kBar + 48, kSFull = kBar + 64, kPFull = kBar + 80;
+    static constexpr int kODone = kBar + 96, kTurn = kBar + 112, kDone = kBar + 128;
+    static constexpr int kTmemSlot = kBar + 136, kAbort = kBar + 140;
+    static constexpr int kBlkIds = kBar + 144;        // int32 [kMaxItemBlocks]
     static constexpr int kRowIdx = kBlkIds + 4 * kMaxItemBlocks;   // int64 [2 * kRows]
     static constexpr int kBytes = kRowIdx + 8 * 2 * kRows;
     static constexpr int kDynSmem = kBytes + 1024;    // room to align the base to 1 KiB
@@ -223,7 +223,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int i = 0; i < 2; ++i) {
             mbar_init(sb + Ly::kKFull + 8 * i, 1);
             mbar_init(sb + Ly::kVFull + 8 * i, 1);
-            mbar_init(sb + Ly::kKvEmpty + 8 * i, 1);
+            mbar_init(sb + Ly::kKEmpty + 8 * i, 1);
+            mbar_init(sb + Ly::kVEmpty + 8 * i, 1);
             mbar_init(sb + Ly::kSFull + 8 * i, 1);
             mbar_init(sb + Ly::kPFull + 8 * i, 128);
             mbar_init(sb + Ly::kODone + 8 * i, 1);
@@ -302,19 +303,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             prefetch_tmap(&tmk);
             prefetch_tmap(&tmv);
-            int issued = 0;
+            int issued = 0, issued_k_only = 0;
             for (int j = 0; j < nkt; ++j) {
                 const int s = j & 1;
-                if (j >= 2 && !wait_bar(sb + Ly::kKvEmpty + 8 * s, ((j >> 1) - 1) & 1, abort)) break;
                 const int b0 = j * 8, nb = min(8, nblk - b0);
                 const uint32_t bytes = (uint32_t)nb * Ly::kHalves * 2048u;
                 const uint32_t kdst = sb + Ly::kK0 + s * Ly::kTile;
                 const uint32_t vdst = sb + Ly::kV0 + s * Ly::kTile;
+                // K(j) may replace K(j-2) once both Q.K MMAs of tile j-2 are
+                // done; V(j) replaces V(j-2) after both P.V MMAs of tile j-2
+                if (j >= 2 && !wait_bar(sb + Ly::kKEmpty + 8 * s, ((j >> 1) - 1) & 1, abort)) break;
                 mbar_arrive_expect_tx(sb + Ly::kKFull + 8 * s, bytes);
                 for (int b = 0; b < nb; ++b)
                     for (int hf = 0; hf < Ly::kHalves; ++hf)
                         tma_load_4d(kdst + hf * Ly::kHalfBytes + b * 2048, &tmk, hf * 64, 0, h,
                                     blk_ids[b0 + b], sb + Ly::kKFull + 8 * s);
+                if (j >= 2 && !wait_bar(sb + Ly::kVEmpty + 8 * s, ((j >> 1) - 1) & 1, abort)) {
+                    issued_k_only = j + 1;
+                    break;
+                }
                 mbar_arrive_expect_tx(sb + Ly::kVFull + 8 * s, bytes);
                 for (int b = 0; b < nb; ++b)
                     for (int hf = 0; hf < Ly::kHalves; ++hf)
@@ -328,13 +335,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_wait(sb + Ly::kKFull + 8 * (j & 1), (j >> 1) & 1, &quiet, kDrainLimitNs);
                 mbar_wait(sb + Ly::kVFull + 8 * (j & 1), (j >> 1) & 1, &quiet, kDrainLimitNs);
             }
+            if (issued_k_only) {
+                const int j = issued_k_only - 1;
+                mbar_wait(sb + Ly::kKFull + 8 * (j & 1), (j >> 1) & 1, &quiet, kDrainLimitNs);
+            }
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         const uint32_t id_qk = idesc_bf16_f32(kRows, kKeys, false);
         const uint32_t id_pv = idesc_bf16_f32(kRows, D, true);
         bool ok = true;
-        // S_X = Q_X . K(j)^T
+        // S_X = Q_X . K(j)^T; the last tile to read K(j) releases its stage
         auto issue_qk = [&](int x, int j) {
             tc_fence_after();
             if (lane == 0) {
@@ -347,6 +358,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                            smem_desc_sw128(kbase + off, 16, 1024), id_qk, kk > 0 ? 1u : 0u);
                 }
                 mma_commit(sb + Ly::kSFull + 8 * x);
+                if (x == 1 || !has_b) mma_commit(sb + Ly::kKEmpty + 8 * (j & 1));
             }
             __syncwarp();
         };
@@ -404,7 +416,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 issue_pv(1, j);
                 if (more) issue_qk(1, j + 1);
             }
-            if (lane == 0) mma_commit(sb + Ly::kKvEmpty + 8 * s);   // K(j), V(j) consumed
+            if (lane == 0) mma_commit(sb + Ly::kVEmpty + 8 * s);    // V(j) consumed
             __syncwarp();
         }
         // all MMAs issued by this thread must finish before TMEM is freed
