@@ -15,6 +15,8 @@ __global__ void __launch_bounds__(256) cache_write_kernel(
     const int64_t *__restrict__ slots, int64_t total_chunks, int32_t chunks_per_token,
     int32_t chunks_per_row, int32_t Hkv, uint4 *__restrict__ k_cache,
     uint4 *__restrict__ v_cache, int64_t num_slots, int *err) {
+    pdl_wait();
+    pdl_trigger();
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < total_chunks; c += stride) {
         const int64_t t = c / chunks_per_token;
@@ -46,12 +48,13 @@ cudaError_t launch_cache_write(const void *k_new, const void *v_new, const int64
     int64_t blocks = (total + 255) / 256;
     if (blocks > 152 * 16) blocks = 152 * 16;
     if (tr) tr->begin(kKernelCacheWrite, stream);
-    cache_write_kernel<<<(unsigned)blocks, 256, 0, stream>>>(
-        reinterpret_cast<const uint4 *>(k_new), reinterpret_cast<const uint4 *>(v_new), slots,
-        total, chunks_per_token, chunks_per_row, Hkv, reinterpret_cast<uint4 *>(k_cache),
-        reinterpret_cast<uint4 *>(v_cache), num_slots, err);
+    cudaError_t e = launch_pdl(cache_write_kernel, dim3((unsigned)blocks), dim3(256), 0, stream,
+                               reinterpret_cast<const uint4 *>(k_new),
+                               reinterpret_cast<const uint4 *>(v_new), slots, total, chunks_per_token,
+                               chunks_per_row, Hkv, reinterpret_cast<uint4 *>(k_cache),
+                               reinterpret_cast<uint4 *>(v_cache), num_slots, err);
     if (tr) tr->end(kKernelCacheWrite, stream);
-    return cudaGetLastError();
+    return e;
 }
 
 }  // namespace pkv

@@ -211,6 +211,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_split_kernel(DecodeArgs a,
                                                                   int32_t num_blocks_pool) {
     extern __shared__ int32_t P[];   // [R + 1]
     __shared__ int32_t s_max_n;
+    pdl_wait();
+    pdl_trigger();
     const int32_t R = lay.R, Hkv = lay.Hkv, Hq = lay.Hq, g = lay.g;
     build_plan(P, R, a.context_lens, a.group_of_req, a.group_blocks, a.num_groups, a.max_blocks,
                &s_max_n, a.err);
@@ -342,14 +344,23 @@ __global__ void __launch_bounds__(kThreads, 1) decode_split_kernel(DecodeArgs a,
     }
 }
 
-// Merge the partials of each (request, q head) with log-sum-exp weights.
+// Merge the partials of each (request, kv head) with log-sum-exp weights:
+// one warp per (request, kv head) merges the g q heads of that kv head, which
+// share one list of parts (the group's prefix splits, then the private
+// pieces).  Lane k holds part k's (m, l) for every head; lane c holds
+// elements [c*E, c*E + E) of every head's output.  All loads of a round are
+// in flight together.
 template <int D>
 __global__ void __launch_bounds__(256) decode_combine_kernel(DecodeArgs a, DecodeLayout lay) {
+    constexpr int E = D / 32;   // output elements per lane and head
+    constexpr int G = 8;        // most q heads per kv head (host-checked)
+    pdl_wait();
+    pdl_trigger();
     const int lane = threadIdx.x & 31;
     const int64_t item = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
-    if (item >= (int64_t)lay.R * lay.Hq) return;
-    const int r = (int)(item / lay.Hq), hq = (int)(item % lay.Hq);
-    const int h = hq / lay.g;
+    if (item >= (int64_t)lay.R * lay.Hkv) return;
+    const int r = (int)(item / lay.Hkv), h = (int)(item % lay.Hkv);
+    const int g = lay.g;
     const float *o_part = reinterpret_cast<const float *>(static_cast<const char *>(a.ws) + lay.off_o);
     const float2 *ml_part =
         reinterpret_cast<const float2 *>(static_cast<const char *>(a.ws) + lay.off_ml);
@@ -364,69 +375,84 @@ __global__ void __launch_bounds__(256) decode_combine_kernel(DecodeArgs a, Decod
             n_pre = min(n_pre, lay.prefix_parts);
         }
     }
-    const int n_priv = min(max(__ldg(nparts + (int64_t)r * lay.Hkv + h), 0), kMaxPrivateParts);
-    const int total = n_pre + n_priv;
-    const int64_t slot0 = item * lay.parts_per_head;
-    auto part_slot = [&](int k) {
-        return slot0 + (k < n_pre ? k : lay.prefix_parts + (k - n_pre));
+    const int n_priv = min(max(__ldg(nparts + item), 0), kMaxPrivateParts);
+    const int total = min(n_pre + n_priv, 32);
+    const int64_t head0 = (int64_t)r * lay.Hq + (int64_t)h * g;   // (request, q head) index of head 0
+    auto part_slot = [&](int hd, int k) {
+        return (head0 + hd) * lay.parts_per_head + (k < n_pre ? k : lay.prefix_parts + (k - n_pre));
     };
-    constexpr int E = D / 32;   // elements per lane
-    constexpr int kRound = 16;  // parts whose loads are in flight together
-    // each lane holds up to two parts' (m, l); issue those loads and the
-    // first round of partial-O loads before using either
-    float2 ml_a = make_float2(-INFINITY, 0.f), ml_b = make_float2(-INFINITY, 0.f);
-    if (lane < total) ml_a = ml_part[part_slot(lane)];
-    if (lane + 32 < total) ml_b = ml_part[part_slot(lane + 32)];
-    float acc[E];
+    // weights: lane k owns part k of every head
+    float wk[G], mx[G], den[G];
 #pragma unroll
-    for (int e = 0; e < E; ++e) acc[e] = 0.f;
-    float mx = 0.f, w_a = 0.f, w_b = 0.f, den = 0.f;
-    for (int k0 = 0; k0 < total; k0 += kRound) {
-        float v[kRound][E];
+    for (int hd = 0; hd < G; ++hd) {
+        float2 v = make_float2(-INFINITY, 0.f);
+        if (hd < g && lane < total) v = ml_part[part_slot(hd, lane)];
+        mx[hd] = v.x;
+        wk[hd] = v.y;   // l for now
+    }
 #pragma unroll
-        for (int u = 0; u < kRound; ++u) {
+    for (int hd = 0; hd < G; ++hd) {
 #pragma unroll
-            for (int e = 0; e < E; ++e) v[u][e] = 0.f;
-            if (k0 + u < total) {
-                const float *src = o_part + part_slot(k0 + u) * D + lane * E;
-                if constexpr (E == 4) {
-                    const float4 t = *reinterpret_cast<const float4 *>(src);
-                    v[u][0] = t.x; v[u][1] = t.y; v[u][2] = t.z; v[u][3] = t.w;
-                } else {
-                    const float2 t = *reinterpret_cast<const float2 *>(src);
-                    v[u][0] = t.x; v[u][1] = t.y;
+        for (int off = 16; off > 0; off >>= 1) mx[hd] = fmaxf(mx[hd], __shfl_xor_sync(0xffffffffu, mx[hd], off));
+    }
+#pragma unroll
+    for (int hd = 0; hd < G; ++hd) {
+        float2 v = make_float2(-INFINITY, 0.f);
+        if (hd < g && lane < total) v = ml_part[part_slot(hd, lane)];
+        const float w = (hd < g && lane < total) ? fast_exp2(v.x - mx[hd]) : 0.f;
+        den[hd] = w * v.y;
+        wk[hd] = w;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) den[hd] += __shfl_xor_sync(0xffffffffu, den[hd], off);
+    }
+    float acc[G][E];
+#pragma unroll
+    for (int hd = 0; hd < G; ++hd)
+#pragma unroll
+        for (int e = 0; e < E; ++e) acc[hd][e] = 0.f;
+    // parts in rounds of KR (KR x G element vectors in flight per lane)
+    constexpr int KR = 2;
+    for (int k0 = 0; k0 < total; k0 += KR) {
+        float v[KR][G][E];
+#pragma unroll
+        for (int u = 0; u < KR; ++u)
+#pragma unroll
+            for (int hd = 0; hd < G; ++hd) {
+#pragma unroll
+                for (int e = 0; e < E; ++e) v[u][hd][e] = 0.f;
+                if (k0 + u < total && hd < g) {
+                    const float *src = o_part + part_slot(hd, k0 + u) * D + lane * E;
+                    if constexpr (E == 4) {
+                        const float4 t = *reinterpret_cast<const float4 *>(src);
+                        v[u][hd][0] = t.x; v[u][hd][1] = t.y; v[u][hd][2] = t.z; v[u][hd][3] = t.w;
+                    } else {
+                        const float2 t = *reinterpret_cast<const float2 *>(src);
+                        v[u][hd][0] = t.x; v[u][hd][1] = t.y;
+                    }
                 }
             }
-        }
-        if (k0 == 0) {
-            mx = fmaxf(ml_a.x, ml_b.x);
 #pragma unroll
-            for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-            w_a = (lane < total) ? fast_exp2(ml_a.x - mx) : 0.f;
-            w_b = (lane + 32 < total) ? fast_exp2(ml_b.x - mx) : 0.f;
-            den = w_a * ml_a.y + w_b * ml_b.y;
+        for (int u = 0; u < KR; ++u)
 #pragma unroll
-            for (int off = 16; off > 0; off >>= 1) den += __shfl_xor_sync(0xffffffffu, den, off);
-        }
+            for (int hd = 0; hd < G; ++hd) {
+                const float w = __shfl_sync(0xffffffffu, wk[hd], (k0 + u) & 31);
 #pragma unroll
-        for (int u = 0; u < kRound; ++u) {
-            const int k = k0 + u;
-            float wk = __shfl_sync(0xffffffffu, k < 32 ? w_a : w_b, k & 31);
-            if (k >= total) wk = 0.f;
-#pragma unroll
-            for (int e = 0; e < E; ++e) acc[e] += wk * v[u][e];
-        }
+                for (int e = 0; e < E; ++e) acc[hd][e] += w * v[u][hd][e];
+            }
     }
-    const float inv = 1.f / den;
-    uint16_t *out = static_cast<uint16_t *>(a.out) + item * D + lane * E;
-    if constexpr (E == 4) {
-        uint2 pk = make_uint2(pack_bf16x2(acc[0] * inv, acc[1] * inv),
-                              pack_bf16x2(acc[2] * inv, acc[3] * inv));
-        *reinterpret_cast<uint2 *>(out) = pk;
-    } else {
-        *reinterpret_cast<uint32_t *>(out) = pack_bf16x2(acc[0] * inv, acc[1] * inv);
+#pragma unroll
+    for (int hd = 0; hd < G; ++hd) {
+        if (hd >= g) break;
+        const float inv = 1.f / den[hd];
+        uint16_t *out = static_cast<uint16_t *>(a.out) + (head0 + hd) * D + lane * E;
+        if constexpr (E == 4) {
+            *reinterpret_cast<uint2 *>(out) = make_uint2(pack_bf16x2(acc[hd][0] * inv, acc[hd][1] * inv),
+                                                         pack_bf16x2(acc[hd][2] * inv, acc[hd][3] * inv));
+        } else {
+            *reinterpret_cast<uint32_t *>(out) = pack_bf16x2(acc[hd][0] * inv, acc[hd][1] * inv);
+        }
+        if (a.lse && lane == 0) a.lse[head0 + hd] = (mx[hd] + __log2f(den[hd])) * 0.69314718055994530942f;
     }
-    if (a.lse && lane == 0) a.lse[item] = (mx + __log2f(den)) * 0.69314718055994530942f;
 }
 
 }  // namespace
@@ -485,16 +511,16 @@ static cudaError_t launch_decode_t(const DecodeLayout &L, const DecodeArgs &a, i
         attr_bytes = smem;
     }
     if (tr) tr->begin(kKernelDecodeSplit, stream);
-    decode_split_kernel<D><<<num_sms, kThreads, smem, stream>>>(a, L, num_blocks_pool);
+    cudaError_t e = launch_pdl(decode_split_kernel<D>, dim3(num_sms), dim3(kThreads), smem, stream,
+                               a, L, num_blocks_pool);
     if (tr) tr->end(kKernelDecodeSplit, stream);
-    cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    const int64_t items = (int64_t)L.R * L.Hq;
+    const int64_t items = (int64_t)L.R * L.Hkv;
     const int64_t grid = (items + 7) / 8;
     if (tr) tr->begin(kKernelDecodeCombine, stream);
-    decode_combine_kernel<D><<<(unsigned)grid, 256, 0, stream>>>(a, L);
+    e = launch_pdl(decode_combine_kernel<D>, dim3((unsigned)grid), dim3(256), 0, stream, a, L);
     if (tr) tr->end(kKernelDecodeCombine, stream);
-    return cudaGetLastError();
+    return e;
 }
 
 cudaError_t launch_decode(const DecodeLayout &L, const DecodeArgs &a, int num_sms,

@@ -27,6 +27,27 @@ struct Tracer {
     virtual ~Tracer() {}
 };
 
+// Launch with programmatic dependent launch allowed: the kernel may be
+// scheduled while its predecessor in the stream is still running; it calls
+// griddepcontrol.wait (pdl_wait) before touching any memory, so it observes
+// everything the predecessor wrote, and releases its own dependent early
+// (pdl_trigger).  This hides the launch latency between the kernels of a step.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t stream, Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 // Set the thread's pkv_last_error() message; returns code.
 int set_last_error(int code, const char *msg);
 
@@ -43,7 +64,7 @@ enum : int {
 // with p in [0, prefix_parts) for the shared-prefix pass and
 // p in [prefix_parts, prefix_parts + kMaxPrivateParts) for private pieces.
 constexpr int kMaxPrivateParts = 16;
-constexpr int kMaxPrefixParts = 48;   // parts_per_head <= 64: two per combine lane
+constexpr int kMaxPrefixParts = 16;   // parts_per_head <= 32: one part per combine lane
 constexpr int kMinBlocksPerPiece = 4;
 
 struct DecodeLayout {

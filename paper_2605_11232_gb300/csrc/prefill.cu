@@ -143,6 +143,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     attn_tile_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
                      const KernelParams p) {
     using Ly = Layout<D>;
+    pdl_wait();
+    pdl_trigger();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int h = blockIdx.x % p.Hkv;
     int nq, nblk, kv_end, q_pos0 = 0, blk_off = 0, cu0 = 0, q0 = 0, m0 = 0;
@@ -637,8 +639,8 @@ static cudaError_t launch_tile_kernel(dim3 grid, const CUtensorMap &tk, const CU
         if (e != cudaSuccess) return e;
         attr = true;
     }
-    attn_tile_kernel<D, PREFIX><<<grid, kThreads, Layout<128>::kDynSmem, stream>>>(tk, tv, p);
-    return cudaGetLastError();
+    return launch_pdl(attn_tile_kernel<D, PREFIX>, grid, dim3(kThreads), Layout<128>::kDynSmem, stream,
+                      tk, tv, p);
 }
 
 cudaError_t launch_prefill(const PrefillArgs &a, cudaStream_t stream, Tracer *tr) {
