@@ -350,10 +350,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_split_kernel(DecodeArgs a,
 // pieces).  Lane k holds part k's (m, l) for every head; lane c holds
 // elements [c*E, c*E + E) of every head's output.  All loads of a round are
 // in flight together.
-template <int D>
+template <int D, int G>
 __global__ void __launch_bounds__(256) decode_combine_kernel(DecodeArgs a, DecodeLayout lay) {
     constexpr int E = D / 32;   // output elements per lane and head
-    constexpr int G = 8;        // most q heads per kv head (host-checked)
+    // G: q heads per kv head rounded up to 4 or 8 (g <= G)
     pdl_wait();
     pdl_trigger();
     const int lane = threadIdx.x & 31;
@@ -411,7 +411,7 @@ __global__ void __launch_bounds__(256) decode_combine_kernel(DecodeArgs a, Decod
 #pragma unroll
         for (int e = 0; e < E; ++e) acc[hd][e] = 0.f;
     // parts in rounds of KR (KR x G element vectors in flight per lane)
-    constexpr int KR = 2;
+    constexpr int KR = 16 / G;
     for (int k0 = 0; k0 < total; k0 += KR) {
         float v[KR][G][E];
 #pragma unroll
@@ -518,7 +518,8 @@ static cudaError_t launch_decode_t(const DecodeLayout &L, const DecodeArgs &a, i
     const int64_t items = (int64_t)L.R * L.Hkv;
     const int64_t grid = (items + 7) / 8;
     if (tr) tr->begin(kKernelDecodeCombine, stream);
-    e = launch_pdl(decode_combine_kernel<D>, dim3((unsigned)grid), dim3(256), 0, stream, a, L);
+    e = L.g <= 4 ? launch_pdl(decode_combine_kernel<D, 4>, dim3((unsigned)grid), dim3(256), 0, stream, a, L)
+                 : launch_pdl(decode_combine_kernel<D, 8>, dim3((unsigned)grid), dim3(256), 0, stream, a, L);
     if (tr) tr->end(kKernelDecodeCombine, stream);
     return e;
 }
