@@ -16,7 +16,6 @@ __global__ void __launch_bounds__(256) cache_write_kernel(
     int32_t chunks_per_row, int32_t Hkv, uint4 *__restrict__ k_cache,
     uint4 *__restrict__ v_cache, int64_t num_slots, int *err) {
     pdl_wait();
-    pdl_trigger();
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < total_chunks; c += stride) {
         const int64_t t = c / chunks_per_token;

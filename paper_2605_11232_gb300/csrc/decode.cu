@@ -212,7 +212,6 @@ __global__ void __launch_bounds__(kThreads, 1) decode_split_kernel(DecodeArgs a,
     extern __shared__ int32_t P[];   // [R + 1]
     __shared__ int32_t s_max_n;
     pdl_wait();
-    pdl_trigger();
     const int32_t R = lay.R, Hkv = lay.Hkv, Hq = lay.Hq, g = lay.g;
     build_plan(P, R, a.context_lens, a.group_of_req, a.group_blocks, a.num_groups, a.max_blocks,
                &s_max_n, a.err);
@@ -355,7 +354,6 @@ __global__ void __launch_bounds__(256) decode_combine_kernel(DecodeArgs a, Decod
     constexpr int E = D / 32;   // output elements per lane and head
     // G: q heads per kv head rounded up to 4 or 8 (g <= G)
     pdl_wait();
-    pdl_trigger();
     const int lane = threadIdx.x & 31;
     const int64_t item = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
     if (item >= (int64_t)lay.R * lay.Hkv) return;

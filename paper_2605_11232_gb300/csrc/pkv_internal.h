@@ -27,11 +27,11 @@ struct Tracer {
     virtual ~Tracer() {}
 };
 
-// Launch with programmatic dependent launch allowed: the kernel may be
-// scheduled while its predecessor in the stream is still running; it calls
-// griddepcontrol.wait (pdl_wait) before touching any memory, so it observes
-// everything the predecessor wrote, and releases its own dependent early
-// (pdl_trigger).  This hides the launch latency between the kernels of a step.
+// Launch with programmatic dependent launch allowed: the kernel's launch is
+// processed while its predecessor in the stream is still running, and its
+// CTAs start as the predecessor's CTAs exit; it calls griddepcontrol.wait
+// (pdl_wait) before touching any memory, so it observes everything the
+// predecessor wrote.  This hides the launch gaps between the kernels of a step.
 template <typename... KArgs, typename... Args>
 cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
                        cudaStream_t stream, Args &&...args) {

@@ -144,7 +144,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                      const KernelParams p) {
     using Ly = Layout<D>;
     pdl_wait();
-    pdl_trigger();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int h = blockIdx.x % p.Hkv;
     int nq, nblk, kv_end, q_pos0 = 0, blk_off = 0, cu0 = 0, q0 = 0, m0 = 0;
