@@ -350,7 +350,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_split_kernel(DecodeArgs a,
 // elements [c*E, c*E + E) of every head's output.  All loads of a round are
 // in flight together.
 template <int D, int G>
-__global__ void __launch_bounds__(256) decode_combine_kernel(DecodeArgs a, DecodeLayout lay) {
+__global__ void __launch_bounds__(128) decode_combine_kernel(DecodeArgs a, DecodeLayout lay) {
     constexpr int E = D / 32;   // output elements per lane and head
     // G: q heads per kv head rounded up to 4 or 8 (g <= G)
     pdl_wait();
@@ -513,11 +513,13 @@ static cudaError_t launch_decode_t(const DecodeLayout &L, const DecodeArgs &a, i
                                a, L, num_blocks_pool);
     if (tr) tr->end(kKernelDecodeSplit, stream);
     if (e != cudaSuccess) return e;
+    // four warps per CTA: small batches spread over more SMs
     const int64_t items = (int64_t)L.R * L.Hkv;
-    const int64_t grid = (items + 7) / 8;
+    const int64_t grid = (items + 3) / 4;
+    if (grid > 0x7fffffff) return cudaErrorInvalidConfiguration;
     if (tr) tr->begin(kKernelDecodeCombine, stream);
-    e = L.g <= 4 ? launch_pdl(decode_combine_kernel<D, 4>, dim3((unsigned)grid), dim3(256), 0, stream, a, L)
-                 : launch_pdl(decode_combine_kernel<D, 8>, dim3((unsigned)grid), dim3(256), 0, stream, a, L);
+    e = L.g <= 4 ? launch_pdl(decode_combine_kernel<D, 4>, dim3((unsigned)grid), dim3(128), 0, stream, a, L)
+                 : launch_pdl(decode_combine_kernel<D, 8>, dim3((unsigned)grid), dim3(128), 0, stream, a, L);
     if (tr) tr->end(kKernelDecodeCombine, stream);
     return e;
 }

@@ -21,12 +21,15 @@
 //              and V from shared memory.
 //   warps 2-3  idle (their warpgroup gives registers to the softmax ones)
 //   warps 4-7  softmax of tile A, warps 8-11 of tile B: thread = row.  S row
-//              from TMEM, causal mask, online max/sum in base 2 (tree
-//              reductions), P (bf16) written back over S in TMEM.  O is
-//              rescaled in TMEM only when the running max grows by more than
-//              2^8; otherwise the stale max is kept (exact: the same max
-//              normalises O and the row sum).  A quarter of the exponentials
-//              run as an FMA-pipe polynomial, the rest on the SFU.
+//              from TMEM, causal mask, online softmax in base 2, P (bf16)
+//              written back over S in TMEM.  After the first key tile one
+//              pass computes P against the running max and the tile's max
+//              together; only when the max grows by more than 2^8 is O
+//              rescaled in TMEM and the pass redone.  Otherwise the stale max
+//              is kept (exact: the same max normalises O and the row sum).
+//              A share of the exponentials runs as an FMA-pipe polynomial,
+//              the rest on the SFU; in the shared-prefix pass the two softmax
+//              warpgroups take turns (see Schedule).
 // Every mbarrier wait is bounded; on a timeout the CTA stops, drains its own
 // TMA copies and MMAs, frees TMEM and latches PKV_ERR_DEVICE_TIMEOUT.
 #include <math.h>
@@ -54,6 +57,13 @@ constexpr uint32_t kTmemCols = 512;   // S_A [0,128) S_B [128,256) O_A [256,384)
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr uint64_t kDrainLimitNs = 200000000ull;
 constexpr int kMaxItemBlocks = 2048;  // keys of one work item <= 32768
+// Softmax schedule per pass: whether the two softmax warpgroups take turns
+// (one group's softmax then overlaps the other group's MMAs instead of
+// sharing issue slots with it), and which share of the exponentials runs on
+// the FMA-pipe polynomial (one pair in kPolyEvery; the rest on the SFU).
+template <bool PREFIX> struct Schedule;
+template <> struct Schedule<false> { static constexpr bool kTurns = false; static constexpr int kPolyEvery = 0; };
+template <> struct Schedule<true> { static constexpr bool kTurns = false; static constexpr int kPolyEvery = 0; };
 
 template <int D>
 struct Layout {
@@ -121,6 +131,52 @@ __device__ __forceinline__ float2 poly_exp2_x2(float2 x) {
                        __uint_as_float(__float_as_uint(t.y) * 0x800000u + __float_as_uint(p.y)));
 }
 
+// Row maximum of the 128 raw scores a thread holds (8 independent chains).
+__device__ __forceinline__ float row_max(const uint32_t (&sr)[4][32]) {
+    float mx8[8];
+#pragma unroll
+    for (int t = 0; t < 8; ++t) mx8[t] = -INFINITY;
+#pragma unroll
+    for (int c = 0; c < 4; ++c)
+#pragma unroll
+        for (int e = 0; e < 32; e += 2)
+            mx8[(e >> 1) & 7] = fmax3(mx8[(e >> 1) & 7], __uint_as_float(sr[c][e]), __uint_as_float(sr[c][e + 1]));
+    return fmaxf(fmax3(mx8[0], mx8[1], mx8[2]), fmax3(fmax3(mx8[3], mx8[4], mx8[5]), mx8[6], mx8[7]));
+}
+
+// One softmax pass over a thread's row of 128 scores: P = 2^(s * scale_log2 -
+// mref) written as bf16 over the row's S columns in TMEM, and the row sum of
+// P returned.  POLY: one pair of exponentials in POLY_EVERY on the FMA-pipe
+// cubic (all inputs finite); otherwise all on the SFU, so masked scores (-inf)
+// give 0.
+// TRACK: also return the scaled row maximum in mx.
+template <bool POLY, bool TRACK, int POLY_EVERY>
+__device__ __forceinline__ float softmax_pass(const uint32_t (&sr)[4][32], float scale_log2, float mref,
+                                              uint32_t s_addr, float &mx) {
+    const float2 sc2 = make_float2(scale_log2, scale_log2);
+    const float2 nm2 = make_float2(-mref, -mref);
+    float2 sum2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+    float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+        uint32_t pk[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+            const float2 sv = make_float2(__uint_as_float(sr[c][2 * e]), __uint_as_float(sr[c][2 * e + 1]));
+            if (TRACK) mx4[e & 3] = fmax3(mx4[e & 3], sv.x, sv.y);
+            const float2 xv = ffma2(sv, sc2, nm2);
+            const float2 pp = (POLY && POLY_EVERY > 0 && (e % (POLY_EVERY > 0 ? POLY_EVERY : 1)) == 1) ? poly_exp2_x2(xv)
+                                                : make_float2(fast_exp2(xv.x), fast_exp2(xv.y));
+            sum2[e & 1] = fadd2(sum2[e & 1], pp);
+            pk[e] = pack_bf16x2(pp.x, pp.y);
+        }
+        tmem_st16(s_addr + c * 16, pk);
+    }
+    if (TRACK) mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * scale_log2;
+    const float2 s2 = fadd2(sum2[0], sum2[1]);
+    return s2.x + s2.y;
+}
+
 __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile int *abort) {
     return mbar_wait(bar, parity, abort, kWaitLimitNs);
 }
@@ -143,6 +199,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     attn_tile_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
                      const KernelParams p) {
     using Ly = Layout<D>;
+    using Sch = Schedule<PREFIX>;
     pdl_wait();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int h = blockIdx.x % p.Hkv;
@@ -183,15 +240,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         nq = min(2 * p.tpt, nm - mt0);
         m0 = gs + mt0;
         // every member id of this item (and the first member, whose table row
-        // names the prefix blocks) must be a request of the batch
-        bool ids_ok = true;
+        // names the prefix blocks) must be a request of the batch: thread i
+        // checks member i (nq <= 256 < kThreads)
         const int r_first = __ldg(p.member_req + gs);
-        if (r_first < 0 || r_first >= p.num_requests) ids_ok = false;
-        for (int i = 0; i < nq; ++i) {
-            const int rm = __ldg(p.member_req + m0 + i);
-            if (rm < 0 || rm >= p.num_requests) ids_ok = false;
+        bool bad = r_first < 0 || r_first >= p.num_requests;
+        if (threadIdx.x < nq) {
+            const int rm = __ldg(p.member_req + m0 + threadIdx.x);
+            bad = bad || rm < 0 || rm >= p.num_requests;
         }
-        if (!ids_ok) {
+        if (__syncthreads_or(bad)) {
             if (threadIdx.x == 0) latch_error(p.err, kDevBounds);
             return;
         }
@@ -257,6 +314,29 @@ __global__ void __launch_bounds__(kThreads, 1)
         blk_ids[b] = id;
     }
     __syncthreads();
+    // The producer issues the K/V loads of the first two key tiles now, so
+    // that their latency overlaps the Q tile loads below.
+    auto issue_kv = [&](int j, bool k_side) {
+        const int s = j & 1;
+        const int b0 = j * 8, nb = min(8, nblk - b0);
+        const uint32_t bytes = (uint32_t)nb * Ly::kHalves * 2048u;
+        const uint32_t bar = sb + (k_side ? Ly::kKFull : Ly::kVFull) + 8 * s;
+        const uint32_t dst = sb + (k_side ? Ly::kK0 : Ly::kV0) + s * Ly::kTile;
+        mbar_arrive_expect_tx(bar, bytes);
+        for (int b = 0; b < nb; ++b)
+            for (int hf = 0; hf < Ly::kHalves; ++hf)
+                tma_load_4d(dst + hf * Ly::kHalfBytes + b * 2048, k_side ? &tmk : &tmv, hf * 64, 0, h,
+                            blk_ids[b0 + b], bar);
+    };
+    const int early = min(2, nkt);
+    if (threadIdx.x == 0) {
+        prefetch_tmap(&tmk);
+        prefetch_tmap(&tmv);
+        for (int j = 0; j < early; ++j) {
+            issue_kv(j, true);
+            issue_kv(j, false);
+        }
+    }
     // Q tiles -> shared memory, K-major with the 128-byte swizzle (16-byte
     // chunk c of row i goes to chunk c ^ (i % 8) of its 128-byte row).  All
     // loads of a round are issued before its first store.
@@ -302,32 +382,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
-            prefetch_tmap(&tmk);
-            prefetch_tmap(&tmv);
-            int issued = 0, issued_k_only = 0;
-            for (int j = 0; j < nkt; ++j) {
+            // key tiles 0 and 1 were issued before the Q load
+            int issued = early, issued_k_only = 0;
+            for (int j = early; j < nkt; ++j) {
                 const int s = j & 1;
-                const int b0 = j * 8, nb = min(8, nblk - b0);
-                const uint32_t bytes = (uint32_t)nb * Ly::kHalves * 2048u;
-                const uint32_t kdst = sb + Ly::kK0 + s * Ly::kTile;
-                const uint32_t vdst = sb + Ly::kV0 + s * Ly::kTile;
                 // K(j) may replace K(j-2) once both Q.K MMAs of tile j-2 are
                 // done; V(j) replaces V(j-2) after both P.V MMAs of tile j-2
-                if (j >= 2 && !wait_bar(sb + Ly::kKEmpty + 8 * s, ((j >> 1) - 1) & 1, abort)) break;
-                mbar_arrive_expect_tx(sb + Ly::kKFull + 8 * s, bytes);
-                for (int b = 0; b < nb; ++b)
-                    for (int hf = 0; hf < Ly::kHalves; ++hf)
-                        tma_load_4d(kdst + hf * Ly::kHalfBytes + b * 2048, &tmk, hf * 64, 0, h,
-                                    blk_ids[b0 + b], sb + Ly::kKFull + 8 * s);
-                if (j >= 2 && !wait_bar(sb + Ly::kVEmpty + 8 * s, ((j >> 1) - 1) & 1, abort)) {
+                if (!wait_bar(sb + Ly::kKEmpty + 8 * s, ((j >> 1) - 1) & 1, abort)) break;
+                issue_kv(j, true);
+                if (!wait_bar(sb + Ly::kVEmpty + 8 * s, ((j >> 1) - 1) & 1, abort)) {
                     issued_k_only = j + 1;
                     break;
                 }
-                mbar_arrive_expect_tx(sb + Ly::kVFull + 8 * s, bytes);
-                for (int b = 0; b < nb; ++b)
-                    for (int hf = 0; hf < Ly::kHalves; ++hf)
-                        tma_load_4d(vdst + hf * Ly::kHalfBytes + b * 2048, &tmv, hf * 64, 0, h,
-                                    blk_ids[b0 + b], sb + Ly::kVFull + 8 * s);
+                issue_kv(j, false);
                 issued = j + 1;
             }
             // let this CTA's own copies land before its shared memory is released
@@ -445,11 +512,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool ok = active;
         for (int j = 0; j < nkt && ok; ++j) {
             if (!warp_wait(sb + Ly::kSFull + 8 * x, j & 1, abort)) { ok = false; break; }
-            // take turns with the other tile's warpgroup, so that one group's
-            // softmax overlaps the other group's MMAs instead of competing for
-            // the same issue slots and SFU (turn[A] is completed by B after
-            // its tile j-1, turn[B] by A after its tile j)
-            if (has_b && (x == 1 || j >= 1) &&
+            // when the schedule says so, take turns with the other tile's
+            // warpgroup (turn[A] is completed by B after its tile j-1, turn[B]
+            // by A after its tile j)
+            if (Sch::kTurns && has_b && (x == 1 || j >= 1) &&
                 !warp_wait(sb + Ly::kTurn + 8 * x, (x ? j : j - 1) & 1, abort)) {
                 ok = false;
                 break;
@@ -461,36 +527,36 @@ __global__ void __launch_bounds__(kThreads, 1)
             tmem_wait_ld();
             const int lim = pos - j * kKeys;          // keys with column index <= lim are visible
             const bool all_visible = __all_sync(0xffffffffu, lim >= kKeys - 1);
-            float mx8[8];
-#pragma unroll
-            for (int t = 0; t < 8; ++t) mx8[t] = -INFINITY;
-            if (all_visible) {
+            if (!all_visible) {
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
 #pragma unroll
-                    for (int e = 0; e < 32; e += 2)
-                        mx8[(e >> 1) & 7] = fmax3(mx8[(e >> 1) & 7], __uint_as_float(sr[c][e]),
-                                                  __uint_as_float(sr[c][e + 1]));
-            } else {
-#pragma unroll
-                for (int c = 0; c < 4; ++c)
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) {
-                        const float v = (c * 32 + e <= lim) ? __uint_as_float(sr[c][e]) : -INFINITY;
-                        sr[c][e] = __float_as_uint(v);
-                        mx8[e & 7] = fmaxf(mx8[e & 7], v);
-                    }
+                    for (int e = 0; e < 32; ++e)
+                        if (c * 32 + e > lim) sr[c][e] = __float_as_uint(-INFINITY);
             }
-            const float mx = fmaxf(fmax3(mx8[0], mx8[1], mx8[2]),
-                                   fmax3(fmax3(mx8[3], mx8[4], mx8[5]), mx8[6], mx8[7])) *
-                             p.scale_log2;            // scale > 0 commutes with max
-            // conditional rescale: keep a stale max unless it grows by > 8 (x256)
-            const float m_new = (mx > m + 8.0f) ? mx : m;
-            const bool grow = (m_new != m) && (j > 0);
-            const float alpha = grow ? fast_exp2(m - m_new) : 1.0f;
-            // P.V(j-1) has completed: Q.K(j), which produced S(j), was issued after it
-            if (__any_sync(0xffffffffu, grow)) {
-#pragma unroll
+            // The first tile finds its row max before the pass.  Later tiles
+            // compute P against the running max m while the pass finds the
+            // tile max; only when some row's max grows by more than 2^8 is O
+            // rescaled and the pass redone with the new max.  (Each pass
+            // variant is instantiated once to keep the loop body small.)
+            if (j == 0) m = row_max(sr) * p.scale_log2;   // scale > 0 commutes with max
+            bool track = j > 0;
+            float tile_sum;
+            for (;;) {
+                float mx = -INFINITY;
+                if (!all_visible)
+                    tile_sum = softmax_pass<false, true, Sch::kPolyEvery>(sr, p.scale_log2, m, s_addr, mx);
+                else if (track)
+                    tile_sum = softmax_pass<true, true, Sch::kPolyEvery>(sr, p.scale_log2, m, s_addr, mx);
+                else
+                    tile_sum = softmax_pass<true, false, Sch::kPolyEvery>(sr, p.scale_log2, m, s_addr, mx);
+                const bool grow = track && mx > m + 8.0f;
+                if (!__any_sync(0xffffffffu, grow)) break;
+                // P.V(j-1) has completed: Q.K(j), which produced S(j), was issued after it
+                const float m_new = grow ? mx : m;
+                const float alpha = grow ? fast_exp2(m - m_new) : 1.0f;
+                tmem_wait_st();
+#pragma unroll 1
                 for (int c = 0; c < D / 32; ++c) {
                     uint32_t o[32];
                     tmem_ld32(o_addr + c * 32, o);
@@ -499,50 +565,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
                     tmem_st32(o_addr + c * 32, o);
                 }
+                l *= alpha;
+                m = m_new;
+                track = false;
             }
-            m = m_new;
-            const float2 sc2 = make_float2(p.scale_log2, p.scale_log2);
-            const float2 nm2 = make_float2(-m, -m);
-            float2 sum2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-            if (all_visible) {
-                // half of the exponentials on the FMA pipe (packed cubic), half on the SFU
-#pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    uint32_t pk[16];
-#pragma unroll
-                    for (int e = 0; e < 16; ++e) {
-                        const float2 xv = ffma2(make_float2(__uint_as_float(sr[c][2 * e]),
-                                                            __uint_as_float(sr[c][2 * e + 1])), sc2, nm2);
-                        const float2 pp = (e & 1) ? poly_exp2_x2(xv)
-                                                  : make_float2(fast_exp2(xv.x), fast_exp2(xv.y));
-                        sum2[e & 1] = fadd2(sum2[e & 1], pp);
-                        pk[e] = pack_bf16x2(pp.x, pp.y);
-                    }
-                    tmem_st16(s_addr + c * 16, pk);
-                }
-            } else {
-                // masked tile: SFU only, so masked scores (-inf) give exactly 0
-#pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    uint32_t pk[16];
-#pragma unroll
-                    for (int e = 0; e < 16; ++e) {
-                        const float2 xv = ffma2(make_float2(__uint_as_float(sr[c][2 * e]),
-                                                            __uint_as_float(sr[c][2 * e + 1])), sc2, nm2);
-                        const float2 pp = make_float2(fast_exp2(xv.x), fast_exp2(xv.y));
-                        sum2[e & 1] = fadd2(sum2[e & 1], pp);
-                        pk[e] = pack_bf16x2(pp.x, pp.y);
-                    }
-                    tmem_st16(s_addr + c * 16, pk);
-                }
-            }
-            const float2 s2 = fadd2(sum2[0], sum2[1]);
-            l = l * alpha + (s2.x + s2.y);
+            l += tile_sum;
             tmem_wait_st();
             tc_fence_before();
             mbar_arrive(sb + Ly::kPFull + 8 * x);
             // hand the turn to the other warpgroup
-            if (has_b && (x == 0 || j + 1 < nkt)) mbar_arrive(sb + Ly::kTurn + 8 * (x ^ 1));
+            if (Sch::kTurns && has_b && (x == 0 || j + 1 < nkt)) mbar_arrive(sb + Ly::kTurn + 8 * (x ^ 1));
         }
         if (ok && warp_wait(sb + Ly::kODone + 8 * x, 0, abort)) {
             tc_fence_after();
