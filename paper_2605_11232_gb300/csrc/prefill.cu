@@ -19,7 +19,7 @@
 //              so the tensor core runs one tile's MMAs while the other tile's
 //              softmax runs.  S = Q.K^T lands in TMEM; P.V reads P from TMEM
 //              and V from shared memory.
-//   warps 2-3  idle (their warpgroup gives registers to the softmax ones)
+//   warps 2-3  idle
 //   warps 4-7  softmax of tile A, warps 8-11 of tile B: thread = row.  S row
 //              from TMEM, causal mask, online softmax in base 2, P (bf16)
 //              written back over S in TMEM.  After the first key tile one
@@ -27,9 +27,11 @@
 //              together; only when the max grows by more than 2^8 is O
 //              rescaled in TMEM and the pass redone.  Otherwise the stale max
 //              is kept (exact: the same max normalises O and the row sum).
-//              A share of the exponentials runs as an FMA-pipe polynomial,
-//              the rest on the SFU; in the shared-prefix pass the two softmax
-//              warpgroups take turns (see Schedule).
+//              The exponentials run on the SFU.  The two softmax warpgroups
+//              run concurrently (their work is staggered by the MMA order).
+// All warps keep the launch allocation of 168 registers: moving registers
+// from the control warps to the softmax warps (setmaxnreg) measured slower,
+// since the MMA issuer then spills in its issue loop.
 // Every mbarrier wait is bounded; on a timeout the CTA stops, drains its own
 // TMA copies and MMAs, frees TMEM and latches PKV_ERR_DEVICE_TIMEOUT.
 #include <math.h>
@@ -45,26 +47,12 @@ namespace {
 using namespace tc;
 
 constexpr int kThreads = 384;
-// launch allocation 168 registers/thread (65536 / 384, rounded to 8); the
-// producer/MMA warpgroup drops to 56 and each softmax warpgroup rises to 224:
-// 56*128 + 2*224*128 = 168*384
-constexpr int kRegsLaunch = 168, kRegsControl = 56, kRegsSoftmax = 224;
-static_assert(kRegsControl * 128 + 2 * kRegsSoftmax * 128 == kRegsLaunch * kThreads,
-              "register split must add up to the launch allocation");
 constexpr int kRows = 128;            // M of one tile
 constexpr int kKeys = 128;            // keys per K/V tile (N of Q.K^T)
 constexpr uint32_t kTmemCols = 512;   // S_A [0,128) S_B [128,256) O_A [256,384) O_B [384,512)
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr uint64_t kDrainLimitNs = 200000000ull;
 constexpr int kMaxItemBlocks = 2048;  // keys of one work item <= 32768
-// Softmax schedule per pass: whether the two softmax warpgroups take turns
-// (one group's softmax then overlaps the other group's MMAs instead of
-// sharing issue slots with it), and which share of the exponentials runs on
-// the FMA-pipe polynomial (one pair in kPolyEvery; the rest on the SFU).
-template <bool PREFIX> struct Schedule;
-template <> struct Schedule<false> { static constexpr bool kTurns = false; static constexpr int kPolyEvery = 0; };
-template <> struct Schedule<true> { static constexpr bool kTurns = false; static constexpr int kPolyEvery = 0; };
-
 template <int D>
 struct Layout {
     static constexpr int kHalves = D / 64;            // 64-element (128-byte) column halves
@@ -75,12 +63,12 @@ struct Layout {
     static constexpr int kV0 = kK0 + 2 * kTile;
     static constexpr int kBar = kV0 + 2 * kTile;
     // barriers: k_full[2] v_full[2] k_empty[2] v_empty[2] s_full[A,B] p_full[A,B]
-    // o_done[A,B] turn[A,B] (the softmax warpgroups take turns) done
+    // o_done[A,B] done
     static constexpr int kKFull = kBar + 0, kVFull = kBar + 16, kKEmpty = kBar + 32;
     static constexpr int kVEmpty = kBar + 48, kSFull = kBar + 64, kPFull = kBar + 80;
-    static constexpr int kODone = kBar + 96, kTurn = kBar + 112, kDone = kBar + 128;
-    static constexpr int kTmemSlot = kBar + 136, kAbort = kBar + 140;
-    static constexpr int kBlkIds = kBar + 144;        // int32 [kMaxItemBlocks]
+    static constexpr int kODone = kBar + 96, kDone = kBar + 112;
+    static constexpr int kTmemSlot = kBar + 120, kAbort = kBar + 124;
+    static constexpr int kBlkIds = kBar + 128;        // int32 [kMaxItemBlocks]
     static constexpr int kRowIdx = kBlkIds + 4 * kMaxItemBlocks;   // int64 [2 * kRows]
     static constexpr int kBytes = kRowIdx + 8 * 2 * kRows;
     static constexpr int kDynSmem = kBytes + 1024;    // room to align the base to 1 KiB
@@ -109,28 +97,6 @@ struct KernelParams {
     float2 *ml_part;            // [R*Hq*parts] (running max (base 2), sum)
 };
 
-// 2^x for two values on the FMA pipe (packed fp32), to offload half of the
-// exponentials from the special-function unit, which alone would need as many
-// cycles per score as the two MMAs take.  x = n + f with n = round(x) found
-// by adding 1.5 * 2^23 (the sum's low mantissa bits hold n), 2^f by a cubic
-// fitted on [-0.5, 0.5] (max relative error 7.5e-5; Lawson-weighted least
-// squares on Chebyshev nodes, see fit_exp2_poly.py), and n added into the
-// exponent field: bits(p) + (n << 23) is one multiply-add on bits(t), since
-// 0x4B400000 << 23 wraps to 0.  x is clamped to -125 so the result stays a
-// normal number; inputs must be finite (masked tiles use the SFU instead).
-__device__ __forceinline__ float2 poly_exp2_x2(float2 x) {
-    const float2 xc = make_float2(fmaxf(x.x, -125.0f), fmaxf(x.y, -125.0f));
-    const float2 t = fadd2(xc, make_float2(12582912.0f, 12582912.0f));
-    const float2 n = fadd2(t, make_float2(-12582912.0f, -12582912.0f));
-    const float2 f = fadd2(xc, make_float2(-n.x, -n.y));
-    float2 p = ffma2(make_float2(0.0551716648f, 0.0551716648f), f,
-                     make_float2(0.2426111251f, 0.2426111251f));
-    p = ffma2(p, f, make_float2(0.6932609677f, 0.6932609677f));
-    p = ffma2(p, f, make_float2(0.9999280572f, 0.9999280572f));
-    return make_float2(__uint_as_float(__float_as_uint(t.x) * 0x800000u + __float_as_uint(p.x)),
-                       __uint_as_float(__float_as_uint(t.y) * 0x800000u + __float_as_uint(p.y)));
-}
-
 // Row maximum of the 128 raw scores a thread holds (8 independent chains).
 __device__ __forceinline__ float row_max(const uint32_t (&sr)[4][32]) {
     float mx8[8];
@@ -145,12 +111,9 @@ __device__ __forceinline__ float row_max(const uint32_t (&sr)[4][32]) {
 }
 
 // One softmax pass over a thread's row of 128 scores: P = 2^(s * scale_log2 -
-// mref) written as bf16 over the row's S columns in TMEM, and the row sum of
-// P returned.  POLY: one pair of exponentials in POLY_EVERY on the FMA-pipe
-// cubic (all inputs finite); otherwise all on the SFU, so masked scores (-inf)
-// give 0.
-// TRACK: also return the scaled row maximum in mx.
-template <bool POLY, bool TRACK, int POLY_EVERY>
+// mref) written as bf16 over the row's S columns in TMEM, the row sum of P
+// returned, and the scaled row maximum left in mx.  Exponentials on the SFU,
+// so masked scores (-inf) give exactly 0.
 __device__ __forceinline__ float softmax_pass(const uint32_t (&sr)[4][32], float scale_log2, float mref,
                                               uint32_t s_addr, float &mx) {
     const float2 sc2 = make_float2(scale_log2, scale_log2);
@@ -163,16 +126,15 @@ __device__ __forceinline__ float softmax_pass(const uint32_t (&sr)[4][32], float
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
             const float2 sv = make_float2(__uint_as_float(sr[c][2 * e]), __uint_as_float(sr[c][2 * e + 1]));
-            if (TRACK) mx4[e & 3] = fmax3(mx4[e & 3], sv.x, sv.y);
+            mx4[e & 3] = fmax3(mx4[e & 3], sv.x, sv.y);
             const float2 xv = ffma2(sv, sc2, nm2);
-            const float2 pp = (POLY && POLY_EVERY > 0 && (e % (POLY_EVERY > 0 ? POLY_EVERY : 1)) == 1) ? poly_exp2_x2(xv)
-                                                : make_float2(fast_exp2(xv.x), fast_exp2(xv.y));
+            const float2 pp = make_float2(fast_exp2(xv.x), fast_exp2(xv.y));
             sum2[e & 1] = fadd2(sum2[e & 1], pp);
             pk[e] = pack_bf16x2(pp.x, pp.y);
         }
         tmem_st16(s_addr + c * 16, pk);
     }
-    if (TRACK) mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * scale_log2;
+    mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * scale_log2;
     const float2 s2 = fadd2(sum2[0], sum2[1]);
     return s2.x + s2.y;
 }
@@ -199,7 +161,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     attn_tile_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
                      const KernelParams p) {
     using Ly = Layout<D>;
-    using Sch = Schedule<PREFIX>;
     pdl_wait();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int h = blockIdx.x % p.Hkv;
@@ -286,7 +247,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(sb + Ly::kSFull + 8 * i, 1);
             mbar_init(sb + Ly::kPFull + 8 * i, 128);
             mbar_init(sb + Ly::kODone + 8 * i, 1);
-            mbar_init(sb + Ly::kTurn + 8 * i, 128);
         }
         mbar_init(sb + Ly::kDone, 1);
         *abort = 0;
@@ -378,7 +338,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem = *tmem_slot;
 
     if (warp < 4) {
-      setmaxnreg_dec<kRegsControl>();
       if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
@@ -494,7 +453,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_wait(sb + Ly::kDone, 0, &quiet, kDrainLimitNs);
       }
     } else {
-        setmaxnreg_inc<kRegsSoftmax>();
         // ------------------------------------------------------------ softmax
         const int x = (warp - 4) >> 2;                // tile A (warps 4-7) or B (8-11)
         const int quarter = warp & 3;                 // TMEM lanes this warp may touch
@@ -512,14 +470,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool ok = active;
         for (int j = 0; j < nkt && ok; ++j) {
             if (!warp_wait(sb + Ly::kSFull + 8 * x, j & 1, abort)) { ok = false; break; }
-            // when the schedule says so, take turns with the other tile's
-            // warpgroup (turn[A] is completed by B after its tile j-1, turn[B]
-            // by A after its tile j)
-            if (Sch::kTurns && has_b && (x == 1 || j >= 1) &&
-                !warp_wait(sb + Ly::kTurn + 8 * x, (x ? j : j - 1) & 1, abort)) {
-                ok = false;
-                break;
-            }
             tc_fence_after();
             uint32_t sr[4][32];
 #pragma unroll
@@ -537,20 +487,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             // The first tile finds its row max before the pass.  Later tiles
             // compute P against the running max m while the pass finds the
             // tile max; only when some row's max grows by more than 2^8 is O
-            // rescaled and the pass redone with the new max.  (Each pass
-            // variant is instantiated once to keep the loop body small.)
+            // rescaled and the pass redone with the new max (after which no
+            // row grows: the redo's tile max is the new max or below m + 8).
             if (j == 0) m = row_max(sr) * p.scale_log2;   // scale > 0 commutes with max
-            bool track = j > 0;
             float tile_sum;
             for (;;) {
-                float mx = -INFINITY;
-                if (!all_visible)
-                    tile_sum = softmax_pass<false, true, Sch::kPolyEvery>(sr, p.scale_log2, m, s_addr, mx);
-                else if (track)
-                    tile_sum = softmax_pass<true, true, Sch::kPolyEvery>(sr, p.scale_log2, m, s_addr, mx);
-                else
-                    tile_sum = softmax_pass<true, false, Sch::kPolyEvery>(sr, p.scale_log2, m, s_addr, mx);
-                const bool grow = track && mx > m + 8.0f;
+                float mx;
+                tile_sum = softmax_pass(sr, p.scale_log2, m, s_addr, mx);
+                const bool grow = j > 0 && mx > m + 8.0f;
                 if (!__any_sync(0xffffffffu, grow)) break;
                 // P.V(j-1) has completed: Q.K(j), which produced S(j), was issued after it
                 const float m_new = grow ? mx : m;
@@ -567,14 +511,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 l *= alpha;
                 m = m_new;
-                track = false;
             }
             l += tile_sum;
             tmem_wait_st();
             tc_fence_before();
             mbar_arrive(sb + Ly::kPFull + 8 * x);
-            // hand the turn to the other warpgroup
-            if (Sch::kTurns && has_b && (x == 0 || j + 1 < nkt)) mbar_arrive(sb + Ly::kTurn + 8 * (x ^ 1));
         }
         if (ok && warp_wait(sb + Ly::kODone + 8 * x, 0, abort)) {
             tc_fence_after();

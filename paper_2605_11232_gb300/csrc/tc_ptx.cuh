@@ -178,18 +178,6 @@ __device__ __forceinline__ void tmem_wait_st() {
 
 // ---- register rebalancing between warpgroups ---------------------------------
 
-// Warpgroup-wide: shrink / grow this warpgroup's per-thread register budget.
-// The increase draws on registers the decreasing warpgroups returned to the
-// CTA's launch allocation.
-template <int N>
-__device__ __forceinline__ void setmaxnreg_dec() {
-    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
-}
-template <int N>
-__device__ __forceinline__ void setmaxnreg_inc() {
-    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
-}
-
 // ---- tcgen05.mma ----------------------------------------------------------------
 
 // Shared-memory matrix descriptor, 128-byte swizzle.  Fields: start address,
