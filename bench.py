@@ -342,9 +342,17 @@ def summarize(res, peaks):
            "ms_range": [min(res["step_ms"]), max(res["step_ms"])],
            "kernels": {k: {"launches": n, "avg_us": 1e3 * t / n} for k, (n, t) in res["trace"].items()}}
     if res["Rd"]:
-        gbs = (res["dec_bytes"] + res["wr_bytes"]) / (ms * 1e-3) / 1e9
+        if res["Rp"]:
+            # mixed step: the decode bytes over the decode kernels' own time
+            # (per-launch CUDA events), not over a step that also runs prefill
+            dec_us = sum(1e3 * t / n for k, (n, t) in res["trace"].items() if k.startswith("decode_"))
+            gbs = res["dec_bytes"] / (dec_us * 1e-6) / 1e9 if dec_us > 0 else float("nan")
+            basis = "decode kernels' CUDA-event time"
+        else:
+            gbs = (res["dec_bytes"] + res["wr_bytes"]) / (ms * 1e-3) / 1e9
+            basis = "whole step (cache write + decode)"
         out.update(decode_hbm_gbs=gbs, decode_frac_of_measured_hbm=gbs / hbm,
-                   decode_frac_of_8tbs=gbs / 8000.0, prefix_pass=res["groups"])
+                   decode_frac_of_8tbs=gbs / 8000.0, decode_basis=basis, prefix_pass=res["groups"])
     if res["Rp"]:
         tp = res["trace"].get("prefill")
         if tp:
