@@ -168,24 +168,42 @@ def barrier(world):
         dist.barrier()
 
 
-def max_over_ranks(x, world):
+def _reduce_over_ranks(x, world, op):
+    """all-reduce one float over the replicas (on the GPU under NCCL, on the
+    CPU under gloo)."""
     if world == 1:
         return x
     import torch
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
-    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=op)
     return float(t.item())
+
+
+def max_over_ranks(x, world):
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    return _reduce_over_ranks(x, world, dist.ReduceOp.MAX)
 
 
 def sum_over_ranks(x, world):
     if world == 1:
         return x
-    import torch
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
-    dist.all_reduce(t, op=dist.ReduceOp.SUM)
-    return float(t.item())
+    return _reduce_over_ranks(x, world, dist.ReduceOp.SUM)
+
+
+def aggregate_replicas(ms_local, step_bytes, e2e_ms_local, world):
+    """Whole-job numbers of N independent replicas: the step time is the
+    slowest rank's, the bytes are every rank's, so value = sum of bytes / max
+    time (weak scaling).  Returns (ms, total_bytes, GB/s, e2e ms, e2e GB/s)."""
+    ms = max_over_ranks(ms_local, world)
+    total_bytes = sum_over_ranks(step_bytes, world)
+    e2e_ms = max_over_ranks(e2e_ms_local, world)
+    return (ms, total_bytes, total_bytes / (ms * 1e-3) / 1e9, e2e_ms,
+            total_bytes / (e2e_ms * 1e-3) / 1e9)
 
 
 def ncu_traffic(kernel: str, workload: str):
@@ -472,12 +490,8 @@ def main():
 
     w = head["w"]
     ms_local = statistics.mean(head["step_ms"])
-    ms = max_over_ranks(ms_local, world)
     step_bytes = head["dec_bytes"] + head["wr_bytes"]
-    total_bytes = sum_over_ranks(step_bytes, world)
-    value = total_bytes / (ms * 1e-3) / 1e9
-    e2e_ms = max_over_ranks(head["e2e_ms"], world)
-    e2e_val = total_bytes / (e2e_ms * 1e-3) / 1e9
+    ms, total_bytes, value, e2e_ms, e2e_val = aggregate_replicas(ms_local, step_bytes, head["e2e_ms"], world)
     hbm, tf_burst, tf_sust, pk_kind = peaks
     # roofline of the dominant kernel (largest share of traced time)
     trace = head["trace"]
