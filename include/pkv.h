@@ -11,8 +11,9 @@
  *
  * Conventions for every call
  *  - All device buffers are owned by the caller.  The library keeps host
- *    metadata (free list, reference counts, TMA descriptors) and one small
- *    device error word per pool, allocated by kv_pool_create.
+ *    metadata (free list, reference counts, TMA descriptors) and 16 bytes of
+ *    device words per pool (an error word and two work counters of the
+ *    decode split pass), allocated by kv_pool_create.
  *  - "device" pointers are CUDA global-memory addresses on the pool's device;
  *    "host" pointers are ordinary CPU memory.  Device buffers must be 16-byte
  *    aligned and contiguous in the stated layout.
@@ -28,6 +29,9 @@
  *    num_q_heads must be a multiple of num_kv_heads; q heads h belong to kv
  *    head h / (num_q_heads / num_kv_heads) (contiguous GQA grouping).
  *  - A pool handle is not thread-safe; calls on one handle must not overlap.
+ *    In particular at most one decode per pool may be in flight on the GPU
+ *    at a time (its split pass takes work from the pool's counters): decodes
+ *    on several streams need one pool each, or an event between them.
  */
 #ifndef PKV_H
 #define PKV_H
@@ -95,12 +99,13 @@ typedef struct {
 /* Create a pool over caller-owned device caches (Sec. 2, Sec. 5.4: paged KV
  * memory).  k_cache/v_cache: device, layout above; both NULL gives a
  * metadata-only pool (allocation calls work, kernel calls fail with
- * PKV_ERR_INVALID_ARG).  On success *out owns host metadata and a 4-byte device
- * error word; free it with kv_pool_destroy.  Errors: INVALID_ARG, UNSUPPORTED
+ * PKV_ERR_INVALID_ARG).  On success *out owns host metadata and 16 bytes of
+ * device words (error word, split-pass counters); free it with
+ * kv_pool_destroy.  Errors: INVALID_ARG, UNSUPPORTED
  * (block_size != 16, head_dim not 64/128, dtype not bf16), CUDA. */
 int kv_pool_create(const pkv_pool_desc *desc, void *k_cache, void *v_cache, pkv_pool_t *out);
 
-/* Free the host metadata and the error word (not the caches).  NULL is a no-op. */
+/* Free the host metadata and the device words (not the caches).  NULL is a no-op. */
 int kv_pool_destroy(pkv_pool_t pool);
 
 /* Take n free blocks; their ids go to ids_out (host, n entries), each with

@@ -27,6 +27,8 @@
 // exactly the keys each thread loaded for P.V.
 #include <math.h>
 
+#include <algorithm>
+
 #include "pkv_device.cuh"
 #include "pkv_internal.h"
 
@@ -36,6 +38,7 @@ namespace {
 
 constexpr int kWarps = 8;
 constexpr int kThreads = kWarps * 32;
+constexpr int kChunksPerWarp = 2;   // work chunks per warp of the grid (balance vs. pipeline restarts)
 
 __device__ __forceinline__ uint32_t reg_of(const uint4 &v, int i) {
     return i == 0 ? v.x : (i == 1 ? v.y : (i == 2 ? v.z : v.w));
@@ -208,25 +211,28 @@ __device__ void build_plan(int32_t *P, int32_t R, const int32_t *__restrict__ co
 
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1) decode_split_kernel(DecodeArgs a, DecodeLayout lay,
-                                                                  int32_t num_blocks_pool) {
+                                                                  int32_t num_blocks_pool,
+                                                                  int32_t after_prefix) {
     extern __shared__ int32_t P[];   // [R + 1]
     __shared__ int32_t s_max_n;
-    pdl_wait();
+    // After a shared-prefix pass, which starts this kernel once it has seen
+    // the cache write complete, nothing read here is written by that pass:
+    // wait for it only before exiting (the combine needs both).  Without one,
+    // wait for the cache write first.
+    if (!after_prefix) pdl_wait();
     const int32_t R = lay.R, Hkv = lay.Hkv, Hq = lay.Hq, g = lay.g;
     build_plan(P, R, a.context_lens, a.group_of_req, a.group_blocks, a.num_groups, a.max_blocks,
                &s_max_n, a.err);
     const int64_t W = (int64_t)Hkv * P[R];
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
-    int64_t per = (W + nwarps - 1) / nwarps;
+    int64_t per = (W + nwarps * kChunksPerWarp - 1) / (nwarps * kChunksPerWarp);
     const int64_t need = (s_max_n - 1 + kMaxPrivateParts - 3) / (kMaxPrivateParts - 2);
     if (per < need) per = need;
     if (per < kMinBlocksPerPiece) per = kMinBlocksPerPiece;
 
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int lr = lane >> 2, lq = lane & 3;
-    const int64_t w = (int64_t)blockIdx.x * kWarps + warp;
-    int64_t x = w * per;
-    const int64_t x_end = min(x + per, W);
+    const int64_t nchunks = (W + per - 1) / per;
 
     const uint16_t *q = static_cast<const uint16_t *>(a.q);
     const uint16_t *kc = static_cast<const uint16_t *>(a.k_cache);
@@ -235,7 +241,16 @@ __global__ void __launch_bounds__(kThreads, 1) decode_split_kernel(DecodeArgs a,
     float2 *ml_part = reinterpret_cast<float2 *>(static_cast<char *>(a.ws) + lay.off_ml);
     int32_t *nparts = reinterpret_cast<int32_t *>(static_cast<char *>(a.ws) + lay.off_nparts);
 
-    while (x < x_end) {
+    // Chunks of `per` stream blocks are handed out by a counter, so that CTAs
+    // which start late (on SMs the prefix pass still holds) take less work.
+    for (;;) {
+      int chunk = 0;
+      if (lane == 0) chunk = atomicAdd(a.sched, 1);
+      chunk = __shfl_sync(0xffffffffu, chunk, 0);
+      if (chunk >= nchunks) break;
+      int64_t x = (int64_t)chunk * per;
+      const int64_t x_end = min(x + per, W);
+      while (x < x_end) {
         // segment containing x: request r (largest r with P[r] <= x / Hkv), head h
         const int64_t xr = x / Hkv;
         int lo = 0, hi = R - 1;
@@ -340,7 +355,14 @@ __global__ void __launch_bounds__(kThreads, 1) decode_split_kernel(DecodeArgs a,
             nparts[(int64_t)r * Hkv + h] = (int32_t)((seg_off + n - 1) / per - seg_off / per + 1);
         }
         x = piece_end;
+      }
     }
+    // the last warp out leaves both counters at zero for the next call
+    if (lane == 0 && atomicAdd(a.sched + 1, 1) == (int)(gridDim.x * kWarps) - 1) {
+        atomicExch(a.sched, 0);
+        atomicExch(a.sched + 1, 0);
+    }
+    if (after_prefix) pdl_wait();
 }
 
 // Merge the partials of each (request, kv head) with log-sum-exp weights:
@@ -460,22 +482,35 @@ DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_
                            int32_t num_sms) {
     DecodeLayout L{};
     L.R = R; L.Hq = Hq; L.Hkv = Hkv; L.d = d; L.g = Hq / Hkv;
+    L.sms = num_sms > 0 ? num_sms : 148;
     L.prefix_blocks_per_part = 8;
     L.prefix_parts = 0;
     if (num_groups > 0 && max_group_blocks > 0 && max_group_members > 0) {
         // Key splits of the prefix pass: one CTA per (group, kv head, member
-        // tile, split), one CTA per SM.  Pick the split count that minimises
-        // waves x (per-CTA set-up + key tiles per CTA), set-up ~ 2 key tiles.
+        // tile, split), one CTA per SM.  The private split pass runs on the
+        // SMs the prefix pass leaves free (it starts as soon as the prefix
+        // pass has), so a step costs about
+        //   max(prefix critical path, (prefix SM-time + split SM-time) / SMs).
+        // Measured on GB300: a prefix CTA costs about 13 us of fixed work
+        // (set-up, Q tile, pipeline fill, partial writes) plus 2.1 us per key
+        // tile; the split pass streams about 41 GB/s per SM.  The private
+        // work is estimated from the table width (60 % of the blocks past the
+        // longest prefix), which only steers the split count.
         const int per_item = 2 * (128 / L.g);   // members per work item (two 128-row tiles)
         const int64_t tiles = (int64_t)num_groups * Hkv * ((max_group_members + per_item - 1) / per_item);
         const int sms = num_sms > 0 ? num_sms : 148;
         const int key_tiles = (max_group_blocks + 7) / 8;
+        const double unit_bytes = 16.0 * d * 2 * 2;   // K + V of one (block, kv head)
+        const double priv_blocks = 0.6 * std::max(1, max_blocks - max_group_blocks);
+        const double split_sm_us = (double)R * Hkv * priv_blocks * unit_bytes / 41e3;
         int best = 1;
-        double best_t = 1e30;
+        double best_t = 1e300;
         for (int sp = 1; sp <= kMaxPrefixParts && sp <= key_tiles; ++sp) {
             const int per = (key_tiles + sp - 1) / sp;
-            const double waves = (double)((tiles * sp + sms - 1) / sms);
-            const double t = waves * (2.0 + per);
+            const int64_t ctas = tiles * sp;
+            const double cta_us = 13.0 + 2.1 * per;
+            const double crit = (double)((ctas + sms - 1) / sms) * cta_us;
+            const double t = std::max(crit, (ctas * cta_us + split_sm_us) / sms);
             if (t < best_t - 1e-9) { best_t = t; best = sp; }
         }
         const int per_tiles = (key_tiles + best - 1) / best;
@@ -489,7 +524,6 @@ DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_
     L.off_ml = up(slots * d * sizeof(float));
     L.off_nparts = L.off_ml + up(slots * sizeof(float2));
     L.total = L.off_nparts + up((size_t)R * Hkv * sizeof(int32_t));
-    (void)max_blocks;
     return L;
 }
 
@@ -509,8 +543,9 @@ static cudaError_t launch_decode_t(const DecodeLayout &L, const DecodeArgs &a, i
         attr_bytes = smem;
     }
     if (tr) tr->begin(kKernelDecodeSplit, stream);
+    const int32_t after_prefix = (L.prefix_parts > 0 && a.num_groups > 0) ? 1 : 0;
     cudaError_t e = launch_pdl(decode_split_kernel<D>, dim3(num_sms), dim3(kThreads), smem, stream,
-                               a, L, num_blocks_pool);
+                               a, L, num_blocks_pool, after_prefix);
     if (tr) tr->end(kKernelDecodeSplit, stream);
     if (e != cudaSuccess) return e;
     // four warps per CTA: small batches spread over more SMs

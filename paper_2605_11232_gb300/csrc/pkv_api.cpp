@@ -79,7 +79,7 @@ struct pkv_pool {
     void *v_cache = nullptr;
     std::vector<int32_t> refcnt;     // 0 = free
     std::vector<int32_t> free_list;  // back() is handed out next
-    int *d_err = nullptr;            // device error word
+    int *d_err = nullptr;            // device words: [0] error, [1..2] decode split scheduling
     int device = -1;
     int num_sms = 0;
     bool tmaps_ready = false;
@@ -217,8 +217,10 @@ int kv_pool_create(const pkv_pool_desc *desc, void *k_cache, void *v_cache, pkv_
     if (k_cache) {
         cudaError_t e = cudaGetDevice(&p->device);
         if (e == cudaSuccess) e = cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount, p->device);
-        if (e == cudaSuccess) e = cudaMalloc(&p->d_err, sizeof(int));
-        if (e == cudaSuccess) e = cudaMemset(p->d_err, 0, sizeof(int));
+        // the error word, then the decode split pass's work and done
+        // counters (zero between calls: the pass's last warp resets them)
+        if (e == cudaSuccess) e = cudaMalloc(&p->d_err, 4 * sizeof(int));
+        if (e == cudaSuccess) e = cudaMemset(p->d_err, 0, 4 * sizeof(int));
         if (e != cudaSuccess) {
             if (p->d_err) cudaFree(p->d_err);
             delete p;
@@ -463,6 +465,7 @@ int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
     }
     a.ws = workspace;
     a.err = pool->d_err;
+    a.sched = pool->d_err + 1;
     a.tmap_k = &pool->tmap_k;
     a.tmap_v = &pool->tmap_v;
     cudaError_t e = pkv::launch_decode(L, a, pool->num_sms, d.num_blocks,

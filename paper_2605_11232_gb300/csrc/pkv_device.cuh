@@ -12,10 +12,16 @@ __device__ __forceinline__ void latch_error(int *err, int code) {
 }
 
 // Programmatic dependent launch: wait until the preceding kernel of the
-// stream has completed and its writes are visible.  Kernels do not trigger
-// their dependents early (the implicit trigger at exit measured faster: an
-// early trigger lets waiting dependent CTAs hold SMs the primary still needs).
+// stream has completed and its writes are visible.  Most kernels let their
+// dependents start only at their exit (the implicit trigger, measured faster
+// than an early one: waiting dependent CTAs would hold SMs the primary still
+// needs).
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Let the next kernel of the stream start now.  The shared-prefix pass does
+// this once it has seen the cache write complete: the private split pass that
+// follows reads nothing the prefix pass writes, so it runs on the SMs the
+// prefix pass leaves free and waits for it only before exiting.
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
 // 16-byte streaming load through the non-coherent path, not kept in L1.
 __device__ __forceinline__ uint4 ldg_stream(const void *p) {

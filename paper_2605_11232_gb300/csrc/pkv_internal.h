@@ -69,6 +69,7 @@ constexpr int kMinBlocksPerPiece = 4;
 
 struct DecodeLayout {
     int32_t R, Hq, Hkv, d, g;
+    int32_t sms;                 // SMs of the device the layout was made for
     int32_t prefix_parts;        // prefix-pass part slots per head (0 without groups)
     int32_t prefix_blocks_per_part;
     int32_t parts_per_head;      // prefix_parts + kMaxPrivateParts
@@ -106,6 +107,7 @@ struct DecodeArgs {
     const int32_t *group_of_req;
     void *ws;
     int *err;
+    int *sched;                  // [0] next chunk, [1] warps done (the split pass)
     const CUtensorMap *tmap_k;   // needed by the shared-prefix pass
     const CUtensorMap *tmap_v;
 };
