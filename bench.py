@@ -313,38 +313,60 @@ def measure_workload(name, steps, warmup, use_groups=True, e2e_steps=0):
                pre_flops=prefill_flops(w, b.pre) if Rp else 0, Rd=Rd, Rp=Rp)
 
     if e2e_steps:
-        # end to end through the C ABI from host buffers: slot mapping on the
-        # host, H2D of the step inputs (pinned), kernels, D2H of the outputs
-        q_h = w.q.pin_memory()
-        k_h = w.new_k.pin_memory()
-        v_h = w.new_v.pin_memory()
-        ctx_h = torch.from_numpy(w.context_lens.astype(np.int32)).pin_memory()
-        slots_h = torch.empty(w.num_new_tokens, dtype=torch.int64).pin_memory()
-        out_dh = torch.empty(out_d.shape, dtype=torch.bfloat16).pin_memory()
-        out_ph = torch.empty(out_p.shape, dtype=torch.bfloat16).pin_memory()
-        h2d = (q_h.numel() * 2 + k_h.numel() * 2 + v_h.numel() * 2 + ctx_h.numel() * 4
-               + slots_h.numel() * 8)
-        d2h = out_dh.numel() * 2 + out_ph.numel() * 2
+        # End to end through the C ABI from host buffers, as a serving loop
+        # runs it: every step computes the slot mapping on the host, copies
+        # the step's inputs (q, new K/V, slots, context lengths) from pinned
+        # memory in one packed H2D copy, runs the kernels and copies the
+        # output back to pinned memory.  Steps are pipelined (the host queues
+        # step i+1 while the GPU runs step i); a pinned buffer is refilled only
+        # after the event of the step that last read it has completed.
+        parts = [("q", b.q), ("k_new", b.k_new), ("v_new", b.v_new), ("slots", b.slots),
+                 ("context_lens", b.context_lens)]
+        offs, n = {}, 0
+        for name, t in parts:
+            offs[name] = n
+            n += (t.numel() * t.element_size() + 255) // 256 * 256
+        dev = torch.empty(n, dtype=torch.uint8, device="cuda")
+        host = [torch.empty(n, dtype=torch.uint8).pin_memory() for _ in range(2)]
 
-        def e2e_step():
-            slots_h.numpy()[:] = pkv.kv_slot_mapping(b.pool, b.table_host, w.context_lens, w.new_lens)
-            b.q.copy_(q_h, non_blocking=True)
-            b.k_new.copy_(k_h, non_blocking=True)
-            b.v_new.copy_(v_h, non_blocking=True)
-            b.context_lens.copy_(ctx_h, non_blocking=True)
-            b.slots.copy_(slots_h, non_blocking=True)
+        def view(buf, name, like):
+            nb = like.numel() * like.element_size()
+            return buf[offs[name]:offs[name] + nb].view(like.dtype).view(like.shape)
+        for hb in host:
+            for name, t in parts:
+                view(hb, name, t).copy_(t.cpu())
+        for name, t in parts:   # the kernels now read the packed buffer
+            v = view(dev, name, t)
+            v.copy_(t)
+            setattr(b, name, v)
+        outs = [t for t in (out_d if Rd else None, out_p if Rp else None) if t is not None]
+        out_h = [[torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in outs] for _ in range(2)]
+        events = [None, None]
+        h2d = n
+        d2h = sum(t.numel() * t.element_size() for t in outs)
+        stream = torch.cuda.current_stream()
+
+        def e2e_step(i):
+            k = i & 1
+            if events[k] is not None:
+                events[k].synchronize()   # the step that last used buffer k is done
+            view(host[k], "slots", b.slots).numpy()[:] = pkv.kv_slot_mapping(
+                b.pool, b.table_host, w.context_lens, w.new_lens)
+            dev.copy_(host[k], non_blocking=True)
             step()
-            if Rd:
-                out_dh.copy_(out_d, non_blocking=True)
-            if Rp:
-                out_ph.copy_(out_p, non_blocking=True)
-            torch.cuda.current_stream().synchronize()
+            for t, th in zip(outs, out_h[k]):
+                th.copy_(t, non_blocking=True)
+            ev = torch.cuda.Event()
+            ev.record(stream)
+            events[k] = ev
 
-        for _ in range(max(3, warmup)):
-            e2e_step()
+        for i in range(max(3, warmup)):
+            e2e_step(i)
+        torch.cuda.synchronize()
         t0 = time.perf_counter()
-        for _ in range(e2e_steps):
-            e2e_step()
+        for i in range(e2e_steps):
+            e2e_step(i)
+        torch.cuda.synchronize()
         t1 = time.perf_counter()
         res.update(e2e_ms=(t1 - t0) * 1e3 / e2e_steps, h2d=h2d, d2h=d2h)
     b.close()
