@@ -72,6 +72,8 @@ struct Layout {
     static constexpr int kRowIdx = kBlkIds + 4 * kMaxItemBlocks;   // int64 [2 * kRows]
     static constexpr int kBytes = kRowIdx + 8 * 2 * kRows;
     static constexpr int kDynSmem = kBytes + 1024;    // room to align the base to 1 KiB
+    // UMMA descriptors hold address / 16 in 14 bits; k-steps add to that field
+    static_assert(kDynSmem < 256 * 1024, "shared addresses must stay below 256 KiB");
 };
 
 struct KernelParams {
@@ -373,44 +375,43 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
+        // Lane 0 alone runs the issue loop: tcgen05.mma and commit are
+        // per-thread, and warp-wide waits and syncs around every group of
+        // MMAs measured 6 % slower on prefill.
+        if (lane == 0) {
         const uint32_t id_qk = idesc_bf16_f32(kRows, kKeys, false);
         const uint32_t id_pv = idesc_bf16_f32(kRows, D, true);
         bool ok = true;
         // S_X = Q_X . K(j)^T; the last tile to read K(j) releases its stage
         auto issue_qk = [&](int x, int j) {
             tc_fence_after();
-            if (lane == 0) {
-                const uint32_t qbase = sb + Ly::kQ + x * Ly::kTile;
-                const uint32_t kbase = sb + Ly::kK0 + (j & 1) * Ly::kTile;
+            // one descriptor per operand tile; a k-step adds its byte offset / 16
+            // to the start-address field (shared addresses < 256 KiB: no carry)
+            const uint64_t qd = smem_desc_sw128(sb + Ly::kQ + x * Ly::kTile, 16, 1024);
+            const uint64_t kd = smem_desc_sw128(sb + Ly::kK0 + (j & 1) * Ly::kTile, 16, 1024);
+            const uint32_t dt = tmem + x * 128;
 #pragma unroll
-                for (int kk = 0; kk < D / 16; ++kk) {
-                    const uint32_t off = (kk >> 2) * Ly::kHalfBytes + (kk & 3) * 32;
-                    mma_ss(tmem + x * 128, smem_desc_sw128(qbase + off, 16, 1024),
-                           smem_desc_sw128(kbase + off, 16, 1024), id_qk, kk > 0 ? 1u : 0u);
-                }
-                mma_commit(sb + Ly::kSFull + 8 * x);
-                if (x == 1 || !has_b) mma_commit(sb + Ly::kKEmpty + 8 * (j & 1));
+            for (int kk = 0; kk < D / 16; ++kk) {
+                const uint32_t off = ((kk >> 2) * Ly::kHalfBytes + (kk & 3) * 32) >> 4;
+                mma_ss(dt, qd + off, kd + off, id_qk, kk > 0 ? 1u : 0u);
             }
-            __syncwarp();
+            mma_commit(sb + Ly::kSFull + 8 * x);
+            if (x == 1 || !has_b) mma_commit(sb + Ly::kKEmpty + 8 * (j & 1));
         };
         // O_X += P_X . V(j)
         auto issue_pv = [&](int x, int j) {
             tc_fence_after();
-            if (lane == 0) {
-                const uint32_t vbase = sb + Ly::kV0 + (j & 1) * Ly::kTile;
+            // V is N-major (head dim contiguous): LBO = stride between the
+            // 64-wide head-dim halves, SBO = stride between 8-key groups; a
+            // 16-key step advances the start address by 2 KiB
+            const uint64_t vd = smem_desc_sw128(sb + Ly::kV0 + (j & 1) * Ly::kTile, Ly::kHalfBytes, 1024);
+            const uint32_t dt = tmem + 256 + x * 128, at = tmem + x * 128;
 #pragma unroll
-                for (int kk = 0; kk < kKeys / 16; ++kk) {
-                    // V is N-major (head dim contiguous): LBO = stride between the
-                    // 64-wide head-dim halves, SBO = stride between 8-key groups
-                    const uint64_t bdesc = smem_desc_sw128(vbase + kk * 2048, Ly::kHalfBytes, 1024);
-                    mma_ts(tmem + 256 + x * 128, tmem + x * 128 + kk * 8, bdesc, id_pv,
-                           (j > 0 || kk > 0) ? 1u : 0u);
-                }
-                if (j == nkt - 1) mma_commit(sb + Ly::kODone + 8 * x);
-            }
-            __syncwarp();
+            for (int kk = 0; kk < kKeys / 16; ++kk)
+                mma_ts(dt, at + kk * 8, vd + (uint64_t)((kk * 2048) >> 4), id_pv, (j > 0 || kk > 0) ? 1u : 0u);
+            if (j == nkt - 1) mma_commit(sb + Ly::kODone + 8 * x);
         };
-        if (warp_wait(sb + Ly::kKFull, 0, abort)) {
+        if (wait_bar(sb + Ly::kKFull, 0, abort)) {
             issue_qk(0, 0);
             if (has_b) issue_qk(1, 0);
         } else {
@@ -418,43 +419,42 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int j = 0; j < nkt && ok; ++j) {
             const int s = j & 1;
-            if (!warp_wait(sb + Ly::kVFull + 8 * s, (j >> 1) & 1, abort)) { ok = false; break; }
+            if (!wait_bar(sb + Ly::kVFull + 8 * s, (j >> 1) & 1, abort)) { ok = false; break; }
             if (j == nkt - 1) {
                 // keys past the item's range: p = 0 there, but their V rows may
                 // hold anything (0 * NaN = NaN in the MMA), so clear them
                 const int first = kv_end - j * kKeys;
                 uint8_t *vs = smem + Ly::kV0 + s * Ly::kTile;
-                for (int row = first + lane; row < kKeys; row += 32)
+                for (int row = first; row < kKeys; ++row)
                     for (int hf = 0; hf < Ly::kHalves; ++hf) {
                         uint4 *d4 = reinterpret_cast<uint4 *>(vs + hf * Ly::kHalfBytes + row * 128);
 #pragma unroll
                         for (int c = 0; c < 8; ++c) d4[c] = make_uint4(0, 0, 0, 0);
                     }
                 fence_proxy_async_smem();
-                __syncwarp();
             }
             const bool more = j + 1 < nkt;
-            if (more && !warp_wait(sb + Ly::kKFull + 8 * (s ^ 1), ((j + 1) >> 1) & 1, abort)) {
+            if (more && !wait_bar(sb + Ly::kKFull + 8 * (s ^ 1), ((j + 1) >> 1) & 1, abort)) {
                 ok = false;
                 break;
             }
             // tile A: P.V(j), then Q.K(j+1) into the S it just consumed
-            if (!warp_wait(sb + Ly::kPFull, j & 1, abort)) { ok = false; break; }
+            if (!wait_bar(sb + Ly::kPFull, j & 1, abort)) { ok = false; break; }
             issue_pv(0, j);
             if (more) issue_qk(0, j + 1);
             if (has_b) {
-                if (!warp_wait(sb + Ly::kPFull + 8, j & 1, abort)) { ok = false; break; }
+                if (!wait_bar(sb + Ly::kPFull + 8, j & 1, abort)) { ok = false; break; }
                 issue_pv(1, j);
                 if (more) issue_qk(1, j + 1);
             }
-            if (lane == 0) mma_commit(sb + Ly::kVEmpty + 8 * s);    // V(j) consumed
-            __syncwarp();
+            mma_commit(sb + Ly::kVEmpty + 8 * s);    // V(j) consumed
         }
         // all MMAs issued by this thread must finish before TMEM is freed
-        if (lane == 0) mma_commit(sb + Ly::kDone);
-        __syncwarp();
+        mma_commit(sb + Ly::kDone);
         int quiet = 0;
         mbar_wait(sb + Ly::kDone, 0, &quiet, kDrainLimitNs);
+        }
+        __syncwarp();
       }
     } else {
         // ------------------------------------------------------------ softmax
