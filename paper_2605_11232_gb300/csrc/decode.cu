@@ -352,7 +352,14 @@ __global__ void __launch_bounds__(kThreads, 1) decode_split_kernel(DecodeArgs a,
             }
         }
         if (x == seg_off && lane == 0) {
-            nparts[(int64_t)r * Hkv + h] = (int32_t)((seg_off + n - 1) / per - seg_off / per + 1);
+            // the segment's part counts for the combine: private pieces in the
+            // low half, the prefix pass's partials of its group in the high one
+            const int32_t n_priv = (int32_t)((seg_off + n - 1) / per - seg_off / per + 1);
+            const int32_t n_pre = lay.prefix_parts > 0 && a.num_groups > 0
+                                      ? min((sh + lay.prefix_blocks_per_part - 1) / lay.prefix_blocks_per_part,
+                                            lay.prefix_parts)
+                                      : 0;
+            nparts[(int64_t)r * Hkv + h] = n_priv | (n_pre << 16);
         }
         x = piece_end;
       }
@@ -386,16 +393,10 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(DecodeArgs a, Decod
         reinterpret_cast<const float2 *>(static_cast<const char *>(a.ws) + lay.off_ml);
     const int32_t *nparts =
         reinterpret_cast<const int32_t *>(static_cast<const char *>(a.ws) + lay.off_nparts);
-    int n_pre = 0;
-    if (a.num_groups > 0) {
-        const int32_t gi = __ldg(a.group_of_req + r);
-        if (gi >= 0 && gi < a.num_groups) {
-            const int32_t gb = __ldg(a.group_blocks + gi);
-            n_pre = (gb + lay.prefix_blocks_per_part - 1) / lay.prefix_blocks_per_part;
-            n_pre = min(n_pre, lay.prefix_parts);
-        }
-    }
-    const int n_priv = min(max(__ldg(nparts + item), 0), kMaxPrivateParts);
+    // part counts written by the split pass: private pieces | prefix partials << 16
+    const int32_t counts = nparts[item];
+    const int n_priv = min(max(counts & 0xFFFF, 0), kMaxPrivateParts);
+    const int n_pre = min((counts >> 16) & 0xFFFF, lay.prefix_parts);
     const int total = min(n_pre + n_priv, 32);
     const int64_t head0 = (int64_t)r * lay.Hq + (int64_t)h * g;   // (request, q head) index of head 0
     auto part_slot = [&](int hd, int k) {

@@ -76,7 +76,7 @@ struct DecodeLayout {
     // byte offsets inside the workspace
     size_t off_o;                // float [R*Hq*parts][d]
     size_t off_ml;               // float2 [R*Hq*parts]
-    size_t off_nparts;           // int32 [R*Hkv] private pieces per (r, kv head)
+    size_t off_nparts;           // int32 [R*Hkv] part counts per (r, kv head): private | prefix << 16
     size_t total;
 };
 
