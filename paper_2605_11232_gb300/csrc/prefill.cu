@@ -23,10 +23,10 @@
 //   warps 4-7  softmax of tile A, warps 8-11 of tile B: thread = row.  S row
 //              from TMEM, causal mask, online softmax in base 2, P (bf16)
 //              written back over S in TMEM.  After the first key tile one
-//              pass computes P against the running max and the tile's max
-//              together; only when the max grows by more than 2^8 is O
-//              rescaled in TMEM and the pass redone.  Otherwise the stale max
-//              is kept (exact: the same max normalises O and the row sum).
+//              pass computes P against the running max, however stale (exact:
+//              the same max normalises O and the row sum); only when the
+//              tile's row sum shows a P above 2^15 is the row max found, O
+//              rescaled in TMEM and the pass redone.
 //              The exponentials run on the SFU.  The two softmax warpgroups
 //              run concurrently (their work is staggered by the MMA order).
 // All warps keep the launch allocation of 168 registers: moving registers
@@ -114,22 +114,19 @@ __device__ __forceinline__ float row_max(const uint32_t (&sr)[4][32]) {
 }
 
 // One softmax pass over a thread's row of 128 scores: P = 2^(s * scale_log2 -
-// mref) written as bf16 over the row's S columns in TMEM, the row sum of P
-// returned, and the scaled row maximum left in mx.  Exponentials on the SFU,
-// so masked scores (-inf) give exactly 0.
+// mref) written as bf16 over the row's S columns in TMEM, and the row sum of
+// P returned.  Exponentials on the SFU, so masked scores (-inf) give exactly 0.
 __device__ __forceinline__ float softmax_pass(const uint32_t (&sr)[4][32], float scale_log2, float mref,
-                                              uint32_t s_addr, float &mx) {
+                                              uint32_t s_addr) {
     const float2 sc2 = make_float2(scale_log2, scale_log2);
     const float2 nm2 = make_float2(-mref, -mref);
     float2 sum2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-    float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
         uint32_t pk[16];
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
             const float2 sv = make_float2(__uint_as_float(sr[c][2 * e]), __uint_as_float(sr[c][2 * e + 1]));
-            mx4[e & 3] = fmax3(mx4[e & 3], sv.x, sv.y);
             const float2 xv = ffma2(sv, sc2, nm2);
             const float2 pp = make_float2(fast_exp2(xv.x), fast_exp2(xv.y));
             sum2[e & 1] = fadd2(sum2[e & 1], pp);
@@ -137,7 +134,6 @@ __device__ __forceinline__ float softmax_pass(const uint32_t (&sr)[4][32], float
         }
         tmem_st16(s_addr + c * 16, pk);
     }
-    mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * scale_log2;
     const float2 s2 = fadd2(sum2[0], sum2[1]);
     return s2.x + s2.y;
 }
@@ -489,20 +485,20 @@ __global__ void __launch_bounds__(kThreads, 1)
                         if (c * 32 + e > lim) sr[c][e] = __float_as_uint(-INFINITY);
             }
             // The first tile finds its row max before the pass.  Later tiles
-            // compute P against the running max m while the pass finds the
-            // tile max; only when some row's max grows by more than 2^8 is O
-            // rescaled and the pass redone with the new max (after which no
-            // row grows: the redo's tile max is the new max or below m + 8).
+            // compute P against the running max m, however stale: the same m
+            // normalises O and the row sum, so the result is exact as long as
+            // no P overflows.  The row sum bounds every P of the tile: a sum
+            // of at most 2^15 means every P <= 2^15 (harmless in bf16 and in
+            // the fp32 accumulators); above it, the row's max is found, O is
+            // rescaled in TMEM and the pass redone with the new max (after
+            // which the sum is at most 128).
             if (j == 0) m = row_max(sr) * p.scale_log2;   // scale > 0 commutes with max
-            float tile_sum;
-            for (;;) {
-                float mx;
-                tile_sum = softmax_pass(sr, p.scale_log2, m, s_addr, mx);
-                const bool grow = j > 0 && mx > m + 8.0f;
-                if (!__any_sync(0xffffffffu, grow)) break;
+            float tile_sum = softmax_pass(sr, p.scale_log2, m, s_addr);
+            const bool grow = tile_sum > 32768.0f;
+            if (__any_sync(0xffffffffu, grow)) {
                 // P.V(j-1) has completed: Q.K(j), which produced S(j), was issued after it
-                const float m_new = grow ? mx : m;
-                const float alpha = grow ? fast_exp2(m - m_new) : 1.0f;
+                const float m_new = grow ? fmaxf(m, row_max(sr) * p.scale_log2) : m;
+                const float alpha = fast_exp2(m - m_new);
                 tmem_wait_st();
 #pragma unroll 1
                 for (int c = 0; c < D / 32; ++c) {
@@ -515,6 +511,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 l *= alpha;
                 m = m_new;
+                tile_sum = softmax_pass(sr, p.scale_log2, m, s_addr);
             }
             l += tile_sum;
             tmem_wait_st();
