@@ -201,3 +201,24 @@ def test_bad_arguments_rejected_before_launch():
         B.run_decode(b, out, None, torch.empty(16, dtype=torch.uint8, device="cuda"), False)
     assert e.value.code == pkv.PKV_ERR_WORKSPACE
     b.close()
+
+
+@pytest.mark.parametrize("groups", [False, True])
+def test_decode_short_and_ragged_segments(groups):
+    """96 requests whose private parts are 1 to 40 blocks (many chunks far
+    shorter than the streaming warps of a CTA, and ragged last blocks), over
+    one shared 256-token prefix and without one: every output against the
+    oracle, no device error."""
+    need_gpu()
+    rng = np.random.default_rng(3)
+    R = 96
+    priv = rng.integers(1, 41 * 16, R)
+    grp = [0 if i % 3 else -1 for i in range(R)]
+    cached = [int(p) - 1 + (256 if g0 == 0 else 0) for p, g0 in zip(priv, grp)]
+    w = make_workload("custom", seed=17, custom=dict(
+        Hq=16, Hkv=2, d=128, prefix_lens=[256], group=grp, cached=cached, new=[1] * R,
+        decode=[True] * R))
+    b = B.build_batch(w, poison=True)
+    out, lse = run_decode(b, use_groups=groups)
+    compare(b, out, lse, range(b.dec.start, b.dec.stop), threads=16)
+    b.close()
