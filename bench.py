@@ -16,6 +16,11 @@ Per-kernel times come from a second pass of K steps with the library's own
 event tracing (pkv_trace_*); the headline pass runs without it, because an
 event between two kernels keeps the second from launching early.
 
+e2e: the headline step driven from pinned host memory through
+paged_attn_decode_step (one H2D copy of the packed inputs, cache write,
+decode, D2H copy of the output), pipelined two steps deep like a serving loop;
+host wall time per step.
+
 --impl reference times the fp64 CPU oracle (the only reference this path has)
 on the host cores, one decode request per step.
 """
@@ -312,50 +317,32 @@ def measure_workload(name, steps, warmup, use_groups=True, e2e_steps=0):
                wr_bytes=write_bytes(w, w.num_new_tokens),
                pre_flops=prefill_flops(w, b.pre) if Rp else 0, Rd=Rd, Rp=Rp)
 
-    if e2e_steps:
+    if e2e_steps and Rd and not Rp:
         # End to end through the C ABI from host buffers, as a serving loop
-        # runs it: every step computes the slot mapping on the host, copies
-        # the step's inputs (q, new K/V, slots, context lengths) from pinned
-        # memory in one packed H2D copy, runs the kernels and copies the
-        # output back to pinned memory.  Steps are pipelined (the host queues
-        # step i+1 while the GPU runs step i); a pinned buffer is refilled only
-        # after the event of the step that last read it has completed.
-        parts = [("q", b.q), ("k_new", b.k_new), ("v_new", b.v_new), ("slots", b.slots),
-                 ("context_lens", b.context_lens)]
-        offs, n = {}, 0
-        for name, t in parts:
-            offs[name] = n
-            n += (t.numel() * t.element_size() + 255) // 256 * 256
-        dev = torch.empty(n, dtype=torch.uint8, device="cuda")
-        host = [torch.empty(n, dtype=torch.uint8).pin_memory() for _ in range(2)]
-
-        def view(buf, name, like):
-            nb = like.numel() * like.element_size()
-            return buf[offs[name]:offs[name] + nb].view(like.dtype).view(like.shape)
-        for hb in host:
-            for name, t in parts:
-                view(hb, name, t).copy_(t.cpu())
-        for name, t in parts:   # the kernels now read the packed buffer
-            v = view(dev, name, t)
-            v.copy_(t)
-            setattr(b, name, v)
-        outs = [t for t in (out_d if Rd else None, out_p if Rp else None) if t is not None]
-        out_h = [[torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in outs] for _ in range(2)]
+        # runs it: every step computes the slot mapping on the host (into the
+        # pinned step buffer), then one paged_attn_decode_step call copies the
+        # step's packed inputs (q, new K/V, slots, context lengths) to the
+        # device, writes the new tokens, decodes and copies the output back to
+        # pinned memory.  Steps are pipelined (the host queues step i+1 while
+        # the GPU runs step i); a pinned buffer is refilled only after the
+        # event of the step that last used it has completed.
+        layout, host, dev = B.step_buffers(b, copies=2)
+        slot_np = [B.step_view(h, layout.slot_mapping, b.slots).numpy() for h in host]
+        out_h = [torch.empty(out_d.shape, dtype=out_d.dtype).pin_memory() for _ in range(2)]
+        steps_k = [pkv.DecodeStep(b.pool, host[k], dev, layout, w.num_new_tokens, b.table[b.dec],
+                                  w.num_q_heads, w.scale, b.groups if groups_ok else None, ws,
+                                  out_d, None, out_h[k], None) for k in range(2)]
         events = [None, None]
-        h2d = n
-        d2h = sum(t.numel() * t.element_size() for t in outs)
+        h2d = layout.bytes
+        d2h = out_d.numel() * out_d.element_size()
         stream = torch.cuda.current_stream()
 
         def e2e_step(i):
             k = i & 1
             if events[k] is not None:
                 events[k].synchronize()   # the step that last used buffer k is done
-            view(host[k], "slots", b.slots).numpy()[:] = pkv.kv_slot_mapping(
-                b.pool, b.table_host, w.context_lens, w.new_lens)
-            dev.copy_(host[k], non_blocking=True)
-            step()
-            for t, th in zip(outs, out_h[k]):
-                th.copy_(t, non_blocking=True)
+            pkv.kv_slot_mapping(b.pool, b.table_host, w.context_lens, w.new_lens, out=slot_np[k])
+            steps_k[k]()
             ev = torch.cuda.Event()
             ev.record(stream)
             events[k] = ev
@@ -368,6 +355,7 @@ def measure_workload(name, steps, warmup, use_groups=True, e2e_steps=0):
             e2e_step(i)
         torch.cuda.synchronize()
         t1 = time.perf_counter()
+        assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
         res.update(e2e_ms=(t1 - t0) * 1e3 / e2e_steps, h2d=h2d, d2h=d2h)
     b.close()
     del b, flush_buf, ws

@@ -217,6 +217,43 @@ int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
                       float scale, const pkv_prefix_groups *groups, void *workspace,
                       size_t workspace_bytes, pkv_stream_t stream);
 
+/* ---- a decode step from host memory --------------------------------------- */
+
+/* Byte offsets of one step's inputs inside a packed buffer, each a multiple
+ * of 16: q bf16 [R][num_q_heads][head_dim], k_new and v_new bf16
+ * [T][num_kv_heads][head_dim], slot_mapping int64 [T], context_lens int32
+ * [R]; bytes = the size of the whole buffer. */
+typedef struct pkv_step_layout {
+    size_t q, k_new, v_new, slot_mapping, context_lens;
+    size_t bytes;
+} pkv_step_layout;
+
+/* One decode step of a serving loop from host memory (Sec. 5.3's decode with
+ * the paged cache of Sec. 5.4), all enqueued on `stream`; the call does not
+ * wait for the GPU:
+ *   1. one copy of layout->bytes bytes from host_in to dev_in (host_in should
+ *      be pinned for the copy to be asynchronous; dev_in is device memory,
+ *      16-byte aligned, with the same layout),
+ *   2. kv_cache_write of the T = num_new_tokens new tokens in dev_in,
+ *   3. paged_attn_decode of the R = num_requests queries in dev_in over
+ *      block_table (device int32 [R][max_blocks]) into out (device bf16) and
+ *      lse (device fp32, or NULL),
+ *   4. a copy of out to host_out, and of lse to host_lse when both are
+ *      non-NULL (host_out may be NULL: no copy).
+ * The caller keeps host_in, host_out and host_lse untouched until the stream
+ * has passed the step (an event recorded after the call).  Other arguments
+ * and the errors are those of kv_cache_write and paged_attn_decode;
+ * INVALID_ARG also for a layout whose regions are misaligned or outside
+ * layout->bytes, CUDA for a failed copy.  The paper has no counterpart: this
+ * composes the entry points above for callers that drive the step from the
+ * host. */
+int paged_attn_decode_step(pkv_pool_t pool, const void *host_in, void *dev_in,
+                           const pkv_step_layout *layout, int32_t num_new_tokens,
+                           const int32_t *block_table, int32_t max_blocks, int32_t num_requests,
+                           int32_t num_q_heads, float scale, const pkv_prefix_groups *groups,
+                           void *workspace, size_t workspace_bytes, void *out, float *lse,
+                           void *host_out, float *host_lse, pkv_stream_t stream);
+
 /* ---- decode without a caller workspace ------------------------------------ */
 
 /* paged_attn_decode for callers that cannot allocate device memory when they

@@ -171,6 +171,40 @@ def build_batch(w: Workload, device="cuda", poison: bool = True, placement_seed=
     return b
 
 
+def step_view(buf: torch.Tensor, off: int, like: torch.Tensor) -> torch.Tensor:
+    """The region of a packed uint8 step buffer at byte offset `off`, viewed
+    with the dtype and shape of `like`."""
+    nb = like.numel() * like.element_size()
+    return buf[off:off + nb].view(like.dtype).view(like.shape)
+
+
+def step_buffers(b: Batch, copies: int = 2):
+    """Packed inputs of one decode step of a decode-only batch (q, new K/V,
+    slot mapping, context lengths; 256-byte aligned regions): the
+    pkv.StepLayout, `copies` pinned host buffers holding them, and a device
+    buffer of the same size."""
+    if b.pre.stop != b.pre.start:
+        raise ValueError("step buffers are for decode-only batches")
+    parts = step_parts(b)
+    offs, n = {}, 0
+    for name, t in parts:
+        offs[name] = n
+        n += (t.numel() * t.element_size() + 255) // 256 * 256
+    layout = pkv.StepLayout(bytes=n, **offs)
+    hosts = [torch.empty(n, dtype=torch.uint8).pin_memory() for _ in range(copies)]
+    for h in hosts:
+        for name, t in parts:
+            step_view(h, offs[name], t).copy_(t.cpu())
+    dev = torch.empty(n, dtype=torch.uint8, device=b.device)
+    return layout, hosts, dev
+
+
+def step_parts(b: Batch):
+    """(field of pkv.StepLayout, device tensor) of a batch's step inputs."""
+    return [("q", b.q), ("k_new", b.k_new), ("v_new", b.v_new), ("slot_mapping", b.slots),
+            ("context_lens", b.context_lens)]
+
+
 def new_token_rows(w: Workload, req: slice) -> slice:
     """Rows of q / k_new belonging to a contiguous request range."""
     return slice(int(w.cu_new[req.start]), int(w.cu_new[req.stop]))

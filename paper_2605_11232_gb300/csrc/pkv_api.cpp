@@ -474,6 +474,57 @@ int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
     return ok();
 }
 
+int paged_attn_decode_step(pkv_pool_t pool, const void *host_in, void *dev_in,
+                           const pkv_step_layout *layout, int32_t num_new_tokens,
+                           const int32_t *block_table, int32_t max_blocks, int32_t num_requests,
+                           int32_t num_q_heads, float scale, const pkv_prefix_groups *groups,
+                           void *workspace, size_t workspace_bytes, void *out, float *lse,
+                           void *host_out, float *host_lse, pkv_stream_t stream) {
+    int rc = check_kernel_pool(pool);
+    if (rc != PKV_OK) return rc;
+    if (!host_in || !dev_in || !layout) return fail(PKV_ERR_INVALID_ARG, "NULL step buffer or layout");
+    if (num_new_tokens < 0 || num_requests < 0 || num_q_heads <= 0)
+        return fail(PKV_ERR_INVALID_ARG, "bad sizes");
+    if (!aligned16(dev_in)) return fail(PKV_ERR_INVALID_ARG, "dev_in must be 16-byte aligned");
+    const pkv_pool_desc &d = pool->desc;
+    const size_t row = (size_t)d.head_dim * 2;
+    // every region 16-byte aligned and inside the buffer
+    const struct { size_t off, len; } regions[] = {
+        {layout->q, (size_t)num_requests * num_q_heads * row},
+        {layout->k_new, (size_t)num_new_tokens * d.num_kv_heads * row},
+        {layout->v_new, (size_t)num_new_tokens * d.num_kv_heads * row},
+        {layout->slot_mapping, (size_t)num_new_tokens * sizeof(int64_t)},
+        {layout->context_lens, (size_t)num_requests * sizeof(int32_t)},
+    };
+    for (const auto &g : regions)
+        if (g.off % 16 != 0 || g.off > layout->bytes || g.len > layout->bytes - g.off)
+            return fail(PKV_ERR_INVALID_ARG, "step layout: region at %zu (%zu bytes) misaligned or "
+                        "outside the %zu-byte buffer", g.off, g.len, layout->bytes);
+    if ((rc = set_device(pool)) != PKV_OK) return rc;
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaMemcpyAsync(dev_in, host_in, layout->bytes, cudaMemcpyHostToDevice, st);
+    if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode_step input copy");
+    const char *din = static_cast<const char *>(dev_in);
+    rc = kv_cache_write(pool, din + layout->k_new, din + layout->v_new,
+                        reinterpret_cast<const int64_t *>(din + layout->slot_mapping), num_new_tokens,
+                        stream);
+    if (rc != PKV_OK) return rc;
+    rc = paged_attn_decode(pool, din + layout->q, out, lse,
+                           reinterpret_cast<const int32_t *>(din + layout->context_lens), block_table,
+                           max_blocks, num_requests, num_q_heads, scale, groups, workspace,
+                           workspace_bytes, stream);
+    if (rc != PKV_OK) return rc;
+    if (host_out && num_requests > 0) {
+        e = cudaMemcpyAsync(host_out, out, (size_t)num_requests * num_q_heads * row,
+                            cudaMemcpyDeviceToHost, st);
+        if (e == cudaSuccess && host_lse && lse)
+            e = cudaMemcpyAsync(host_lse, lse, (size_t)num_requests * num_q_heads * sizeof(float),
+                                cudaMemcpyDeviceToHost, st);
+        if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode_step output copy");
+    }
+    return ok();
+}
+
 int pkv_check_device_errors(pkv_pool_t pool, pkv_stream_t stream, int32_t *code_out) {
     int rc = check_kernel_pool(pool);
     if (rc != PKV_OK) return rc;

@@ -32,8 +32,8 @@ EXPORTS = [
     "kv_pool_create", "kv_pool_destroy", "kv_pool_alloc", "kv_pool_retain", "kv_pool_release",
     "kv_pool_refcount", "kv_pool_num_free", "kv_pool_alloc_sequence", "kv_slot_mapping",
     "kv_cache_write", "paged_attn_prefill", "paged_attn_decode_workspace_size",
-    "paged_attn_decode", "paged_attn_decode_noalloc", "pkv_trace_enable", "pkv_trace_read", "pkv_check_device_errors",
-    "pkv_last_error",
+    "paged_attn_decode", "paged_attn_decode_noalloc", "paged_attn_decode_step", "pkv_trace_enable",
+    "pkv_trace_read", "pkv_check_device_errors", "pkv_last_error",
 ]
 
 
@@ -60,6 +60,13 @@ class PrefixGroups(ctypes.Structure):
                 ("max_group_members", ctypes.c_int32), ("reserved", ctypes.c_int32),
                 ("group_start", ctypes.c_void_p), ("member_req", ctypes.c_void_p),
                 ("group_blocks", ctypes.c_void_p), ("group_of_req", ctypes.c_void_p)]
+
+
+class StepLayout(ctypes.Structure):
+    """Byte offsets of one decode step's inputs in a packed buffer (pkv_step_layout)."""
+    _fields_ = [("q", ctypes.c_size_t), ("k_new", ctypes.c_size_t), ("v_new", ctypes.c_size_t),
+                ("slot_mapping", ctypes.c_size_t), ("context_lens", ctypes.c_size_t),
+                ("bytes", ctypes.c_size_t)]
 
 
 _lib = None
@@ -96,6 +103,8 @@ def load(path: str | None = None):
         "pkv_check_device_errors": [V, V, P],
         "paged_attn_decode_noalloc": [V, V, V, V, V, V, i32, i32, i32, f32,
                                       ctypes.POINTER(PrefixGroups), V],
+        "paged_attn_decode_step": [V, V, V, ctypes.POINTER(StepLayout), i32, V, i32, i32, i32, f32,
+                                   ctypes.POINTER(PrefixGroups), V, sz, V, V, V, V, V],
         "pkv_trace_enable": [V, i32],
         "pkv_trace_read": [V, P, i32, P],
     }
@@ -192,14 +201,21 @@ def kv_pool_alloc_sequence(pool, prefix_ids, n_blocks: int) -> np.ndarray:
 
 # ---- a2: slot mapping --------------------------------------------------------
 
-def kv_slot_mapping(pool, block_table: np.ndarray, context_lens, new_lens) -> np.ndarray:
+def kv_slot_mapping(pool, block_table: np.ndarray, context_lens, new_lens,
+                    out: np.ndarray | None = None) -> np.ndarray:
+    """Slots of the new tokens; written into ``out`` (contiguous int64, one per
+    new token) when given, e.g. a view of a pinned step buffer."""
     table = np.ascontiguousarray(block_table, np.int32)
     ctx = np.ascontiguousarray(context_lens, np.int32)
     new = np.ascontiguousarray(new_lens, np.int32)
-    out = np.zeros(max(int(new.sum()), 1), np.int64)
+    n = int(new.sum())
+    if out is None:
+        out = np.zeros(max(n, 1), np.int64)
+    elif out.dtype != np.int64 or not out.flags.c_contiguous or out.size < n:
+        raise ValueError("out must be a contiguous int64 array with one entry per new token")
     _check(load().kv_slot_mapping(pool, _np_ptr(table), table.shape[1], _np_ptr(ctx),
                                   _np_ptr(new), len(ctx), _np_ptr(out)))
-    return out[: int(new.sum())]
+    return out[:n]
 
 
 # ---- a3-a7: kernels ---------------------------------------------------------
@@ -250,6 +266,54 @@ def paged_attn_decode_noalloc(pool, q, out, lse, context_lens, block_table, scal
         pool, _dptr(q), _dptr(out), _dptr(lse), _dptr(context_lens), _dptr(block_table),
         int(block_table.shape[1]), int(context_lens.shape[0]), int(q.shape[1]), float(scale),
         ctypes.byref(groups) if groups is not None else None, _stream(stream)))
+
+
+def _hptr(t):
+    """Address of a host (CPU) torch tensor, or None."""
+    if t is None:
+        return None
+    if t.is_cuda or not t.is_contiguous():
+        raise ValueError("expected a contiguous CPU tensor")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _step_args(pool, host_in, dev_in, layout, num_new_tokens, block_table, num_q_heads, scale,
+               groups, workspace, out, lse, host_out, host_lse, stream):
+    return (pool, _hptr(host_in), _dptr(dev_in), ctypes.byref(layout), int(num_new_tokens),
+            _dptr(block_table), int(block_table.shape[1]), int(block_table.shape[0]),
+            int(num_q_heads), float(scale), ctypes.byref(groups) if groups is not None else None,
+            _dptr(workspace),
+            int(workspace.numel() * workspace.element_size()) if workspace is not None else 0,
+            _dptr(out), _dptr(lse), _hptr(host_out), _hptr(host_lse), _stream(stream))
+
+
+def paged_attn_decode_step(pool, host_in, dev_in, layout: StepLayout, num_new_tokens: int,
+                           block_table, num_q_heads: int, scale: float, groups, workspace, out,
+                           lse=None, host_out=None, host_lse=None, stream=None):
+    """One decode step from a packed host buffer (pinned uint8 CPU tensor):
+    H2D copy, cache write, decode, D2H copy of the output; enqueued, not
+    waited for."""
+    _check(load().paged_attn_decode_step(*_step_args(
+        pool, host_in, dev_in, layout, num_new_tokens, block_table, num_q_heads, scale, groups,
+        workspace, out, lse, host_out, host_lse, stream)))
+
+
+class DecodeStep:
+    """paged_attn_decode_step with its arguments converted once, for a serving
+    loop that calls it every step on the same buffers (keeps them alive)."""
+
+    def __init__(self, pool, host_in, dev_in, layout: StepLayout, num_new_tokens: int,
+                 block_table, num_q_heads: int, scale: float, groups, workspace, out, lse=None,
+                 host_out=None, host_lse=None, stream=None):
+        self._keep = (host_in, dev_in, layout, block_table, groups, workspace, out, lse, host_out,
+                      host_lse)
+        self._args = _step_args(pool, host_in, dev_in, layout, num_new_tokens, block_table,
+                                num_q_heads, scale, groups, workspace, out, lse, host_out,
+                                host_lse, stream)
+        self._fn = load().paged_attn_decode_step
+
+    def __call__(self):
+        _check(self._fn(*self._args))
 
 
 def pkv_trace_enable(pool, enable: bool = True):

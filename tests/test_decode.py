@@ -222,3 +222,39 @@ def test_decode_short_and_ragged_segments(groups):
     out, lse = run_decode(b, use_groups=groups)
     compare(b, out, lse, range(b.dec.start, b.dec.stop), threads=16)
     b.close()
+
+
+@pytest.mark.parametrize("groups", [False, True])
+def test_decode_step_from_host_buffers_bit_exact(groups):
+    """paged_attn_decode_step (one H2D copy of the packed inputs, cache write,
+    decode, D2H copy of the output) gives the bits of kv_cache_write +
+    paged_attn_decode on device inputs, on two steps in a row."""
+    need_gpu()
+    w = make_workload("l8b_decode", scale_requests=0.25)
+    b = B.build_batch(w, poison=True)
+    ref, ref_lse = run_decode(b, use_groups=groups)
+    layout, hosts, dev = B.step_buffers(b, copies=1)
+    R = b.dec.stop - b.dec.start
+    ws = B.decode_workspace(b, groups)
+    out = torch.empty_like(ref)
+    lse = torch.empty_like(ref_lse)
+    host_out = torch.full(tuple(ref.shape), float("nan"), dtype=torch.bfloat16).pin_memory()
+    host_lse = torch.full((R, w.num_q_heads), float("nan"), dtype=torch.float32).pin_memory()
+    step = pkv.DecodeStep(b.pool, hosts[0], dev, layout, w.num_new_tokens, b.table[b.dec],
+                          w.num_q_heads, w.scale, b.groups if groups else None, ws, out, lse,
+                          host_out, host_lse)
+    for _ in range(2):
+        host_out.fill_(float("nan"))
+        step()
+        torch.cuda.synchronize()
+        assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
+        assert torch.equal(host_out, ref.cpu()) and torch.equal(host_lse, ref_lse.cpu())
+    # a misaligned region is refused before anything is enqueued
+    bad = pkv.StepLayout(q=layout.q, k_new=layout.k_new + 8, v_new=layout.v_new,
+                         slot_mapping=layout.slot_mapping, context_lens=layout.context_lens,
+                         bytes=layout.bytes)
+    with pytest.raises(pkv.PkvError) as e:
+        pkv.paged_attn_decode_step(b.pool, hosts[0], dev, bad, w.num_new_tokens, b.table[b.dec],
+                                   w.num_q_heads, w.scale, None, ws, out)
+    assert e.value.code == pkv.PKV_ERR_INVALID_ARG
+    b.close()
