@@ -18,8 +18,9 @@ event between two kernels keeps the second from launching early.
 
 e2e: the headline step driven from pinned host memory through
 paged_attn_decode_step (one H2D copy of the packed inputs, cache write,
-decode, D2H copy of the output), pipelined two steps deep like a serving loop;
-host wall time per step.
+decode, D2H copy of the output), alternate steps on two streams so that one
+step's copies overlap the other's kernels, like a serving loop; host wall time
+per step.
 
 --impl reference times the fp64 CPU oracle (the only reference this path has)
 on the host cores, one decode request per step.
@@ -323,19 +324,29 @@ def measure_workload(name, steps, warmup, use_groups=True, e2e_steps=0):
         # pinned step buffer), then one paged_attn_decode_step call copies the
         # step's packed inputs (q, new K/V, slots, context lengths) to the
         # device, writes the new tokens, decodes and copies the output back to
-        # pinned memory.  Steps are pipelined (the host queues step i+1 while
-        # the GPU runs step i); a pinned buffer is refilled only after the
-        # event of the step that last used it has completed.
-        layout, host, dev = B.step_buffers(b, copies=2)
+        # pinned memory.  Alternate steps go to two streams, each with its own
+        # device input and output buffers; a step's kernels wait for the
+        # previous step's (one decode per pool at a time), so its copies
+        # overlap the other stream's kernels.  A pinned buffer is refilled
+        # only after the step that last used it has completed.
+        layout, host, _ = B.step_buffers(b, copies=2)
         slot_np = [B.step_view(h, layout.slot_mapping, b.slots).numpy() for h in host]
+        dev = [torch.empty(layout.bytes, dtype=torch.uint8, device=b.device) for _ in range(2)]
+        for k in range(2):
+            dev[k].copy_(host[k])
+        outs = [torch.empty_like(out_d) for _ in range(2)]
         out_h = [torch.empty(out_d.shape, dtype=out_d.dtype).pin_memory() for _ in range(2)]
-        steps_k = [pkv.DecodeStep(b.pool, host[k], dev, layout, w.num_new_tokens, b.table[b.dec],
-                                  w.num_q_heads, w.scale, b.groups if groups_ok else None, ws,
-                                  out_d, None, out_h[k], None) for k in range(2)]
+        streams = [torch.cuda.Stream() for _ in range(2)]
+        done = [torch.cuda.Event() for _ in range(2)]
+        steps_k = [pkv.DecodeStep(b.pool, host[k], dev[k], layout, w.num_new_tokens,
+                                  b.table[b.dec], w.num_q_heads, w.scale,
+                                  b.groups if groups_ok else None, ws, outs[k], None, out_h[k],
+                                  None, wait_event=done[1 - k], done_event=done[k],
+                                  stream=streams[k]) for k in range(2)]
+        torch.cuda.synchronize()
         events = [None, None]
         h2d = layout.bytes
         d2h = out_d.numel() * out_d.element_size()
-        stream = torch.cuda.current_stream()
 
         def e2e_step(i):
             k = i & 1
@@ -344,7 +355,7 @@ def measure_workload(name, steps, warmup, use_groups=True, e2e_steps=0):
             pkv.kv_slot_mapping(b.pool, b.table_host, w.context_lens, w.new_lens, out=slot_np[k])
             steps_k[k]()
             ev = torch.cuda.Event()
-            ev.record(stream)
+            ev.record(streams[k])
             events[k] = ev
 
         for i in range(max(3, warmup)):
@@ -356,6 +367,7 @@ def measure_workload(name, steps, warmup, use_groups=True, e2e_steps=0):
         torch.cuda.synchronize()
         t1 = time.perf_counter()
         assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
+        assert torch.equal(out_h[0], out_h[1])   # every step computes the same batch
         res.update(e2e_ms=(t1 - t0) * 1e3 / e2e_steps, h2d=h2d, d2h=d2h)
     b.close()
     del b, flush_buf, ws

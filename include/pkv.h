@@ -45,6 +45,7 @@ extern "C" {
 
 typedef struct pkv_pool *pkv_pool_t;
 typedef void *pkv_stream_t; /* a cudaStream_t */
+typedef void *pkv_event_t;  /* a cudaEvent_t */
 
 typedef enum {
     PKV_OK = 0,
@@ -240,6 +241,13 @@ typedef struct pkv_step_layout {
  *      lse (device fp32, or NULL),
  *   4. a copy of out to host_out, and of lse to host_lse when both are
  *      non-NULL (host_out may be NULL: no copy).
+ * wait_event (a cudaEvent_t, or NULL): the kernels wait for it after the
+ * input copy.  done_event (or NULL): recorded once the kernels are done,
+ * before the output copy.  With two streams taking alternate steps, each
+ * with its own dev_in, out and lse, and each step waiting for the previous
+ * step's done_event, a step's copies overlap the other stream's kernels
+ * while the kernels themselves stay in order (at most one decode per pool in
+ * flight).
  * The caller keeps host_in, host_out and host_lse untouched until the stream
  * has passed the step (an event recorded after the call).  Other arguments
  * and the errors are those of kv_cache_write and paged_attn_decode;
@@ -252,7 +260,8 @@ int paged_attn_decode_step(pkv_pool_t pool, const void *host_in, void *dev_in,
                            const int32_t *block_table, int32_t max_blocks, int32_t num_requests,
                            int32_t num_q_heads, float scale, const pkv_prefix_groups *groups,
                            void *workspace, size_t workspace_bytes, void *out, float *lse,
-                           void *host_out, float *host_lse, pkv_stream_t stream);
+                           void *host_out, float *host_lse, pkv_event_t wait_event,
+                           pkv_event_t done_event, pkv_stream_t stream);
 
 /* ---- decode without a caller workspace ------------------------------------ */
 

@@ -479,7 +479,8 @@ int paged_attn_decode_step(pkv_pool_t pool, const void *host_in, void *dev_in,
                            const int32_t *block_table, int32_t max_blocks, int32_t num_requests,
                            int32_t num_q_heads, float scale, const pkv_prefix_groups *groups,
                            void *workspace, size_t workspace_bytes, void *out, float *lse,
-                           void *host_out, float *host_lse, pkv_stream_t stream) {
+                           void *host_out, float *host_lse, pkv_event_t wait_event,
+                           pkv_event_t done_event, pkv_stream_t stream) {
     int rc = check_kernel_pool(pool);
     if (rc != PKV_OK) return rc;
     if (!host_in || !dev_in || !layout) return fail(PKV_ERR_INVALID_ARG, "NULL step buffer or layout");
@@ -504,6 +505,10 @@ int paged_attn_decode_step(pkv_pool_t pool, const void *host_in, void *dev_in,
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     cudaError_t e = cudaMemcpyAsync(dev_in, host_in, layout->bytes, cudaMemcpyHostToDevice, st);
     if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode_step input copy");
+    if (wait_event) {
+        e = cudaStreamWaitEvent(st, static_cast<cudaEvent_t>(wait_event), 0);
+        if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode_step wait_event");
+    }
     const char *din = static_cast<const char *>(dev_in);
     rc = kv_cache_write(pool, din + layout->k_new, din + layout->v_new,
                         reinterpret_cast<const int64_t *>(din + layout->slot_mapping), num_new_tokens,
@@ -514,6 +519,10 @@ int paged_attn_decode_step(pkv_pool_t pool, const void *host_in, void *dev_in,
                            max_blocks, num_requests, num_q_heads, scale, groups, workspace,
                            workspace_bytes, stream);
     if (rc != PKV_OK) return rc;
+    if (done_event) {
+        e = cudaEventRecord(static_cast<cudaEvent_t>(done_event), st);
+        if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode_step done_event");
+    }
     if (host_out && num_requests > 0) {
         e = cudaMemcpyAsync(host_out, out, (size_t)num_requests * num_q_heads * row,
                             cudaMemcpyDeviceToHost, st);

@@ -104,7 +104,7 @@ def load(path: str | None = None):
         "paged_attn_decode_noalloc": [V, V, V, V, V, V, i32, i32, i32, f32,
                                       ctypes.POINTER(PrefixGroups), V],
         "paged_attn_decode_step": [V, V, V, ctypes.POINTER(StepLayout), i32, V, i32, i32, i32, f32,
-                                   ctypes.POINTER(PrefixGroups), V, sz, V, V, V, V, V],
+                                   ctypes.POINTER(PrefixGroups), V, sz, V, V, V, V, V, V, V],
         "pkv_trace_enable": [V, i32],
         "pkv_trace_read": [V, P, i32, P],
     }
@@ -277,25 +277,37 @@ def _hptr(t):
     return ctypes.c_void_p(t.data_ptr())
 
 
+def _event(ev):
+    """cudaEvent_t of a torch.cuda.Event (created on first use), or None."""
+    if ev is None:
+        return None
+    if ev.cuda_event == 0:
+        ev.record()   # torch creates the CUDA event lazily, at its first record
+    return ctypes.c_void_p(ev.cuda_event)
+
+
 def _step_args(pool, host_in, dev_in, layout, num_new_tokens, block_table, num_q_heads, scale,
-               groups, workspace, out, lse, host_out, host_lse, stream):
+               groups, workspace, out, lse, host_out, host_lse, wait_event, done_event, stream):
     return (pool, _hptr(host_in), _dptr(dev_in), ctypes.byref(layout), int(num_new_tokens),
             _dptr(block_table), int(block_table.shape[1]), int(block_table.shape[0]),
             int(num_q_heads), float(scale), ctypes.byref(groups) if groups is not None else None,
             _dptr(workspace),
             int(workspace.numel() * workspace.element_size()) if workspace is not None else 0,
-            _dptr(out), _dptr(lse), _hptr(host_out), _hptr(host_lse), _stream(stream))
+            _dptr(out), _dptr(lse), _hptr(host_out), _hptr(host_lse), _event(wait_event),
+            _event(done_event), _stream(stream))
 
 
 def paged_attn_decode_step(pool, host_in, dev_in, layout: StepLayout, num_new_tokens: int,
                            block_table, num_q_heads: int, scale: float, groups, workspace, out,
-                           lse=None, host_out=None, host_lse=None, stream=None):
+                           lse=None, host_out=None, host_lse=None, wait_event=None,
+                           done_event=None, stream=None):
     """One decode step from a packed host buffer (pinned uint8 CPU tensor):
-    H2D copy, cache write, decode, D2H copy of the output; enqueued, not
-    waited for."""
+    H2D copy, [wait for wait_event], cache write, decode, [record done_event],
+    D2H copy of the output; enqueued, not waited for.  Events are
+    torch.cuda.Event objects."""
     _check(load().paged_attn_decode_step(*_step_args(
         pool, host_in, dev_in, layout, num_new_tokens, block_table, num_q_heads, scale, groups,
-        workspace, out, lse, host_out, host_lse, stream)))
+        workspace, out, lse, host_out, host_lse, wait_event, done_event, stream)))
 
 
 class DecodeStep:
@@ -304,12 +316,12 @@ class DecodeStep:
 
     def __init__(self, pool, host_in, dev_in, layout: StepLayout, num_new_tokens: int,
                  block_table, num_q_heads: int, scale: float, groups, workspace, out, lse=None,
-                 host_out=None, host_lse=None, stream=None):
+                 host_out=None, host_lse=None, wait_event=None, done_event=None, stream=None):
         self._keep = (host_in, dev_in, layout, block_table, groups, workspace, out, lse, host_out,
-                      host_lse)
+                      host_lse, wait_event, done_event, stream)
         self._args = _step_args(pool, host_in, dev_in, layout, num_new_tokens, block_table,
                                 num_q_heads, scale, groups, workspace, out, lse, host_out,
-                                host_lse, stream)
+                                host_lse, wait_event, done_event, stream)
         self._fn = load().paged_attn_decode_step
 
     def __call__(self):

@@ -258,3 +258,31 @@ def test_decode_step_from_host_buffers_bit_exact(groups):
                                    w.num_q_heads, w.scale, None, ws, out)
     assert e.value.code == pkv.PKV_ERR_INVALID_ARG
     b.close()
+
+
+def test_decode_step_two_streams_alternating():
+    """Alternate steps on two streams, each with its own device input and
+    output buffers, each step's kernels waiting for the previous step's
+    done_event: every step's host output has the device path's bits."""
+    need_gpu()
+    w = make_workload("l8b_decode", scale_requests=0.25)
+    b = B.build_batch(w, poison=True)
+    ref, _ = run_decode(b, use_groups=True)
+    layout, hosts, _ = B.step_buffers(b, copies=2)
+    ws = B.decode_workspace(b, True)
+    devs = [torch.empty(layout.bytes, dtype=torch.uint8, device="cuda") for _ in range(2)]
+    outs = [torch.empty_like(ref) for _ in range(2)]
+    streams = [torch.cuda.Stream() for _ in range(2)]
+    done = [torch.cuda.Event() for _ in range(2)]
+    host_outs = [torch.empty(tuple(ref.shape), dtype=torch.bfloat16).pin_memory() for _ in range(4)]
+    for i in range(4):
+        k = i & 1
+        pkv.paged_attn_decode_step(b.pool, hosts[k], devs[k], layout, w.num_new_tokens,
+                                   b.table[b.dec], w.num_q_heads, w.scale, b.groups, ws, outs[k],
+                                   host_out=host_outs[i], wait_event=done[1 - k],
+                                   done_event=done[k], stream=streams[k])
+    torch.cuda.synchronize()
+    assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
+    for h in host_outs:
+        assert torch.equal(h, ref.cpu())
+    b.close()
