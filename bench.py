@@ -292,6 +292,8 @@ def measure_workload(name, steps, warmup, use_groups=True, e2e_steps=0):
         step()
     torch.cuda.synchronize()
     step_ms = run_steps(step, flush, steps, stream)
+    # the same steps back to back with no flush (warm L2), reported beside
+    warm_ms = run_steps(step, lambda: None, steps, stream)
     # traced pass (per-kernel CUDA events from the library) for the roofline
     pkv.pkv_trace_enable(b.pool, True)
     for _ in range(min(warmup, 3)):
@@ -313,7 +315,8 @@ def measure_workload(name, steps, warmup, use_groups=True, e2e_steps=0):
         kb["decode_split"] = (rows_priv + (0 if groups_ok else rows_pre)) * kv_row_bytes(w) + qo
         kb["decode_prefix"] = rows_pre * kv_row_bytes(w) + qo if groups_ok else 0
         kb["decode_combine"] = qo
-    res = dict(name=name, w=w, step_ms=step_ms, trace=trace, groups=groups_ok, kernel_bytes=kb,
+    res = dict(name=name, w=w, step_ms=step_ms, warm_ms=warm_ms, trace=trace, groups=groups_ok,
+               kernel_bytes=kb,
                dec_bytes=decode_bytes(w, b.dec) if Rd else 0,
                wr_bytes=write_bytes(w, w.num_new_tokens),
                pre_flops=prefill_flops(w, b.pre) if Rp else 0, Rd=Rd, Rp=Rp)
@@ -380,6 +383,7 @@ def summarize(res, peaks):
     ms = statistics.mean(res["step_ms"])
     out = {"ms_per_step": ms, "ms_median": statistics.median(res["step_ms"]),
            "ms_range": [min(res["step_ms"]), max(res["step_ms"])],
+           "ms_per_step_warm_l2": statistics.mean(res["warm_ms"]),
            "kernels": {k: {"launches": n, "avg_us": 1e3 * t / n} for k, (n, t) in res["trace"].items()}}
     if res["Rd"]:
         if res["Rp"]:
@@ -393,6 +397,9 @@ def summarize(res, peaks):
             basis = "whole step (cache write + decode)"
         out.update(decode_hbm_gbs=gbs, decode_frac_of_measured_hbm=gbs / hbm,
                    decode_frac_of_8tbs=gbs / 8000.0, decode_basis=basis, prefix_pass=res["groups"])
+        if not res["Rp"]:
+            out["decode_hbm_gbs_warm_l2"] = (res["dec_bytes"] + res["wr_bytes"]) / (
+                statistics.mean(res["warm_ms"]) * 1e-3) / 1e9
     if res["Rp"]:
         tp = res["trace"].get("prefill")
         if tp:
@@ -458,10 +465,23 @@ def cpu_baseline(w_name, budget_s=12.0):
         if time.perf_counter() - t0 > budget_s:
             break
     dt = time.perf_counter() - t0
+    # the same oracle on one thread, over the first requests for about a
+    # quarter of the budget
+    t1 = time.perf_counter()
+    n1 = 0
+    for r in range(w.num_requests):
+        oracle.request_attention(w, r, threads=1)
+        n1 += 1
+        if time.perf_counter() - t1 > budget_s / 4:
+            break
+    dt1 = time.perf_counter() - t1
     return {"value": done * per_pass / dt / 1e9, "unit": "GB/s", "cores": cores, "kind": "oracle",
             "sample": f"{done} passes over all {w.num_requests} {w_name} decode requests (all q heads, "
                       f"full context), fp64 C oracle, {cores} threads, {dt:.1f} s; bytes counted like "
-                      "the GPU metric (shared prefix once per pass)"}
+                      "the GPU metric (shared prefix once per pass)",
+            "one_thread": {"value": per_pass * n1 / w.num_requests / dt1 / 1e9, "unit": "GB/s",
+                           "sample": f"{n1} of the {w.num_requests} requests on 1 thread, {dt1:.1f} s; "
+                                     "bytes: the pass's, in proportion to the requests done"}}
 
 
 def main():

@@ -153,6 +153,51 @@ int kv_slot_mapping(pkv_pool_t pool, const int32_t *block_table, int32_t max_blo
                     const int32_t *context_lens, const int32_t *new_lens, int32_t num_requests,
                     int64_t *slots_out);
 
+/* ---- automatic prefix caching (host) -------------------------------------- */
+
+/* An index of cached full blocks of a pool, keyed by token prefix: the prefix
+ * reuse of Automatic Prefix Caching (Sec. 5.4).  A request's tokens are cut
+ * into blocks of 16; a full block is keyed by its whole token prefix (its own
+ * 16 tokens and all before them).  The index holds one reference on every
+ * block it caches, so a cached block outlives the request that wrote it;
+ * blocks that only the index holds are evicted least recently used first.
+ * Keys are chained 64-bit hashes checked token by token, so a collision never
+ * shares a block.  Host only; a handle is not thread-safe, and the pool must
+ * outlive it. */
+typedef struct pkv_prefix_cache *pkv_prefix_cache_t;
+
+/* flags for pkv_prefix_cache_create: test aid that keeps 4 bits of every key,
+ * so that most lookups meet colliding keys. */
+#define PKV_PREFIX_CACHE_WEAK_HASH 1
+
+int pkv_prefix_cache_create(pkv_pool_t pool, int32_t flags, pkv_prefix_cache_t *out);
+/* Drops the index's reference on every cached block. NULL is a no-op. */
+int pkv_prefix_cache_destroy(pkv_prefix_cache_t cache);
+/* The longest run of cached full blocks that begins tokens[0 .. n_tokens):
+ * their ids (at most max_ids) go to ids_out[0 .. *n_ids_out), each retained
+ * once more for the caller's request (refcount + 1), so they can head its
+ * block-table row; the rest of the row comes from kv_pool_alloc, and the
+ * request releases the whole row when it ends.  Marks them used. */
+int pkv_prefix_cache_match(pkv_prefix_cache_t cache, const int32_t *tokens, int32_t n_tokens,
+                           int32_t *ids_out, int32_t max_ids, int32_t *n_ids_out);
+/* Register the full blocks of tokens[0 .. n_tokens) held in ids[0 .. n_ids)
+ * (block j holds tokens [16j, 16j + 16); the caller holds every id and has
+ * written its K/V).  A block whose prefix is not cached yet is added and
+ * retained by the index; a prefix already cached keeps its block.  Every
+ * block of the path is marked used.  *n_added_out (may be NULL) counts the
+ * new entries.  Errors: REFCOUNT for a free id, INVALID_ARG. */
+int pkv_prefix_cache_insert(pkv_prefix_cache_t cache, const int32_t *tokens, int32_t n_tokens,
+                            const int32_t *ids, int32_t n_ids, int32_t *n_added_out);
+/* Evict up to n_wanted cached blocks that no request holds (the index's
+ * reference is the only one) and whose cached successors are gone: least
+ * recently used first, then the deeper block, then the older entry.  Each is
+ * released to the pool's free list; their ids go to ids_out[0 ..
+ * *n_evicted_out). */
+int pkv_prefix_cache_evict(pkv_prefix_cache_t cache, int32_t n_wanted, int32_t *ids_out,
+                           int32_t *n_evicted_out);
+/* Number of cached blocks. */
+int pkv_prefix_cache_size(pkv_prefix_cache_t cache, int32_t *n_cached_out);
+
 /* ---- a3: cache write (device) ------------------------------------------- */
 
 /* Scatter new-token keys and values into their slots (bit-exact copy).

@@ -33,7 +33,9 @@ EXPORTS = [
     "kv_pool_refcount", "kv_pool_num_free", "kv_pool_alloc_sequence", "kv_slot_mapping",
     "kv_cache_write", "paged_attn_prefill", "paged_attn_decode_workspace_size",
     "paged_attn_decode", "paged_attn_decode_noalloc", "paged_attn_decode_step", "pkv_trace_enable",
-    "pkv_trace_read", "pkv_check_device_errors", "pkv_last_error",
+    "pkv_trace_read", "pkv_check_device_errors", "pkv_last_error", "pkv_prefix_cache_create",
+    "pkv_prefix_cache_destroy", "pkv_prefix_cache_match", "pkv_prefix_cache_insert",
+    "pkv_prefix_cache_evict", "pkv_prefix_cache_size",
 ]
 
 
@@ -106,6 +108,12 @@ def load(path: str | None = None):
         "paged_attn_decode_step": [V, V, V, ctypes.POINTER(StepLayout), i32, V, i32, i32, i32, f32,
                                    ctypes.POINTER(PrefixGroups), V, sz, V, V, V, V, V, V, V],
         "pkv_trace_enable": [V, i32],
+        "pkv_prefix_cache_create": [V, i32, ctypes.POINTER(V)],
+        "pkv_prefix_cache_destroy": [V],
+        "pkv_prefix_cache_match": [V, P, i32, P, i32, P],
+        "pkv_prefix_cache_insert": [V, P, i32, P, i32, P],
+        "pkv_prefix_cache_evict": [V, i32, P, P],
+        "pkv_prefix_cache_size": [V, P],
         "pkv_trace_read": [V, P, i32, P],
     }
     for name, args in sig.items():
@@ -326,6 +334,56 @@ class DecodeStep:
 
     def __call__(self):
         _check(self._fn(*self._args))
+
+
+# ---- automatic prefix caching (host) ----------------------------------------
+
+PKV_PREFIX_CACHE_WEAK_HASH = 1
+
+
+def pkv_prefix_cache_create(pool, weak_hash: bool = False):
+    h = ctypes.c_void_p()
+    _check(load().pkv_prefix_cache_create(pool, PKV_PREFIX_CACHE_WEAK_HASH if weak_hash else 0,
+                                          ctypes.byref(h)))
+    return h
+
+
+def pkv_prefix_cache_destroy(cache):
+    _check(load().pkv_prefix_cache_destroy(cache))
+
+
+def pkv_prefix_cache_match(cache, tokens, max_ids: int | None = None) -> np.ndarray:
+    """Ids of the longest run of cached full blocks heading `tokens` (each
+    retained once more for the caller)."""
+    t = np.ascontiguousarray(tokens, np.int32)
+    cap = len(t) // 16 if max_ids is None else int(max_ids)
+    out = np.zeros(max(cap, 1), np.int32)
+    n = np.zeros(1, np.int32)
+    _check(load().pkv_prefix_cache_match(cache, _np_ptr(t), len(t), _np_ptr(out), cap, _np_ptr(n)))
+    return out[: int(n[0])]
+
+
+def pkv_prefix_cache_insert(cache, tokens, ids) -> int:
+    """Register the full blocks of `tokens` held in `ids`; returns the number
+    of new entries."""
+    t = np.ascontiguousarray(tokens, np.int32)
+    i = np.ascontiguousarray(ids, np.int32)
+    n = np.zeros(1, np.int32)
+    _check(load().pkv_prefix_cache_insert(cache, _np_ptr(t), len(t), _np_ptr(i), len(i), _np_ptr(n)))
+    return int(n[0])
+
+
+def pkv_prefix_cache_evict(cache, n_wanted: int) -> np.ndarray:
+    out = np.zeros(max(int(n_wanted), 1), np.int32)
+    n = np.zeros(1, np.int32)
+    _check(load().pkv_prefix_cache_evict(cache, int(n_wanted), _np_ptr(out), _np_ptr(n)))
+    return out[: int(n[0])]
+
+
+def pkv_prefix_cache_size(cache) -> int:
+    n = np.zeros(1, np.int32)
+    _check(load().pkv_prefix_cache_size(cache, _np_ptr(n)))
+    return int(n[0])
 
 
 def pkv_trace_enable(pool, enable: bool = True):
