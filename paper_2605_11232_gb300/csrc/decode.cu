@@ -230,7 +230,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_split_kernel(DecodeArgs a,
     if (per < need) per = need;
     if (per < kMinBlocksPerPiece) per = kMinBlocksPerPiece;
 
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
     const int lr = lane >> 2, lq = lane & 3;
     const int64_t nchunks = (W + per - 1) / per;
 
