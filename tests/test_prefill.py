@@ -180,3 +180,23 @@ def test_prefill_causality_future_keys_ignored():
         assert torch.equal(o1[a:e - 1], o2[a:e - 1]) and torch.equal(l1[a:e - 1], l2[a:e - 1])
         assert not torch.equal(o1[e - 1], o2[e - 1])
     b.close()
+
+
+def test_speculative_verify_chain_drafts():
+    """Verification of k = 2..8 chain draft tokens per request (each draft
+    attends to the whole context and to the drafts before it) is a suffix
+    prefill with S = k: 16 requests, 12 of them over one shared 512-token
+    prefix, ragged private contexts; every row against the oracle."""
+    need_gpu()
+    rng = np.random.default_rng(8)
+    R = 16
+    k = [2 + (i % 7) for i in range(R)]
+    grp = [0 if i % 4 else -1 for i in range(R)]
+    cached = [int(rng.integers(1, 40 * 16)) + (512 if g0 == 0 else 0) for g0 in grp]
+    w = make_workload("custom", seed=9, custom=dict(
+        Hq=32, Hkv=8, d=128, prefix_lens=[512], group=grp, cached=cached, new=k,
+        decode=[False] * R))
+    b = B.build_batch(w, poison=True)
+    out, lse = run_prefill(b)
+    compare(b, out, lse, range(R))
+    b.close()
