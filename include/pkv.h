@@ -9,6 +9,14 @@
  * (Automatic Prefix Caching, Sec. 2 and Sec. 5.4; the design rule at the end
  * of Sec. 3 that shared prefixes are not recomputed).
  *
+ * Contents: the block pool and its reference counts (kv_pool_*), slot
+ * mapping (kv_slot_mapping), the prefix-caching index (pkv_prefix_cache_*),
+ * the cache write (kv_cache_write), suffix prefill (paged_attn_prefill),
+ * decode (paged_attn_decode; without a caller workspace:
+ * paged_attn_decode_noalloc; one host-driven step with its copies:
+ * paged_attn_decode_step), per-kernel tracing (pkv_trace_*) and device error
+ * reporting (pkv_check_device_errors).
+ *
  * Conventions for every call
  *  - All device buffers are owned by the caller.  The library keeps host
  *    metadata (free list, reference counts, TMA descriptors) and 16 bytes of
