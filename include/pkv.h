@@ -10,7 +10,8 @@
  * of Sec. 3 that shared prefixes are not recomputed).
  *
  * Contents: the block pool and its reference counts (kv_pool_*), slot
- * mapping (kv_slot_mapping), the prefix-caching index (pkv_prefix_cache_*),
+ * mapping (kv_slot_mapping), the prefix-caching index (pkv_prefix_cache_*)
+ * and the prefix groups of a decode batch (pkv_prefix_groups_build),
  * the cache write (kv_cache_write), suffix prefill (paged_attn_prefill),
  * decode (paged_attn_decode; without a caller workspace:
  * paged_attn_decode_noalloc; one host-driven step with its copies:
@@ -205,6 +206,28 @@ int pkv_prefix_cache_evict(pkv_prefix_cache_t cache, int32_t n_wanted, int32_t *
                            int32_t *n_evicted_out);
 /* Number of cached blocks. */
 int pkv_prefix_cache_size(pkv_prefix_cache_t cache, int32_t *n_cached_out);
+
+/* Prefix groups of a decode batch from its block tables (host; the
+ * descriptor that paged_attn_decode's shared-prefix pass takes): requests
+ * whose rows begin with the same physical blocks, e.g. blocks handed out by
+ * pkv_prefix_cache_match, share those blocks.  Rule: candidates are grouped
+ * by their first block id (in request order).  A member's shareable run is
+ * the run of equal leading ids it has with the group's first candidate,
+ * capped at (context_lens[r] - 1) / 16 blocks so that the block holding its
+ * query token stays private; candidates whose run is shorter than
+ * min_shared_blocks (>= 1) stay out; the group shares the shortest run of
+ * its members; groups of one member are dropped (their request gets -1).
+ *  block_table: host int32 [R][max_blocks]; context_lens: host int32 [R].
+ *  Outputs (host): group_of_req_out [R] (-1: no group), group_start_out
+ *  [R + 1] (CSR offsets into member_req_out; G + 1 used), member_req_out [R],
+ *  group_blocks_out [R] (G used), *num_groups_out = G, and the largest group
+ *  blocks and member counts. */
+int pkv_prefix_groups_build(const int32_t *block_table, int32_t max_blocks, int32_t num_requests,
+                            const int32_t *context_lens, int32_t min_shared_blocks,
+                            int32_t *group_of_req_out, int32_t *group_start_out,
+                            int32_t *member_req_out, int32_t *group_blocks_out,
+                            int32_t *num_groups_out, int32_t *max_group_blocks_out,
+                            int32_t *max_group_members_out);
 
 /* ---- a3: cache write (device) ------------------------------------------- */
 

@@ -104,3 +104,44 @@ class PrefixCacheModel:
 
     def size(self):
         return len(self.entries)
+
+
+def prefix_groups(table, context_lens, min_shared_blocks=1):
+    """Prefix groups of a decode batch, written out: candidates (requests with
+    at least min_shared_blocks shareable blocks, i.e. (L - 1) // 16 full
+    blocks before the one holding the query) grouped by their first block id
+    in order of first appearance; a member's run is its run of equal leading
+    ids with the group's first candidate, within its cap; candidates below
+    min_shared_blocks stay out; a group of at least two shares the shortest
+    run.  Returns (group_of_req, [(members, shared_blocks), ...])."""
+    R, mb = len(table), len(table[0]) if len(table) else 0
+    cap = [min((int(L) - 1) // BS, mb) if L >= 1 else 0 for L in context_lens]
+    order, cand = [], {}
+    for r in range(R):
+        if cap[r] < min_shared_blocks or table[r][0] < 0:
+            continue
+        f = int(table[r][0])
+        if f not in cand:
+            cand[f] = []
+            order.append(f)
+        cand[f].append(r)
+    group_of_req = [-1] * R
+    groups = []
+    for f in order:
+        c = cand[f]
+        if len(c) < 2:
+            continue
+        ref = table[c[0]]
+        runs = []
+        for r in c:
+            k = 0
+            while k < cap[r] and table[r][k] == ref[k] and table[r][k] >= 0:
+                k += 1
+            if k >= min_shared_blocks:
+                runs.append((r, k))
+        if len(runs) < 2:
+            continue
+        for r, _ in runs:
+            group_of_req[r] = len(groups)
+        groups.append(([r for r, _ in runs], min(k for _, k in runs)))
+    return group_of_req, groups

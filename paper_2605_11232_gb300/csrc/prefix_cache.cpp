@@ -244,3 +244,69 @@ int pkv_prefix_cache_size(pkv_prefix_cache_t cache, int32_t *n_cached_out) {
 }
 
 }  // extern "C"
+
+// ---- prefix groups of a decode batch ----------------------------------------
+
+extern "C" int pkv_prefix_groups_build(const int32_t *block_table, int32_t max_blocks,
+                                       int32_t num_requests, const int32_t *context_lens,
+                                       int32_t min_shared_blocks, int32_t *group_of_req_out,
+                                       int32_t *group_start_out, int32_t *member_req_out,
+                                       int32_t *group_blocks_out, int32_t *num_groups_out,
+                                       int32_t *max_group_blocks_out,
+                                       int32_t *max_group_members_out) {
+    if (num_requests < 0 || max_blocks <= 0 || min_shared_blocks < 1 || !num_groups_out ||
+        !max_group_blocks_out || !max_group_members_out ||
+        (num_requests > 0 && (!block_table || !context_lens || !group_of_req_out || !group_start_out ||
+                              !member_req_out || !group_blocks_out)))
+        return fail(PKV_ERR_INVALID_ARG, "bad arguments");
+    *num_groups_out = *max_group_blocks_out = *max_group_members_out = 0;
+    if (num_requests == 0) return PKV_OK;
+    group_start_out[0] = 0;
+    const int32_t R = num_requests;
+    auto row = [&](int32_t r) { return block_table + (size_t)r * max_blocks; };
+    // blocks of request r that may be shared: full blocks before the one that
+    // holds its query token (a decode request keeps at least one private block)
+    auto cap = [&](int32_t r) {
+        const int32_t L = context_lens[r];
+        return L < 1 ? 0 : std::min((L - 1) / kBlock, max_blocks);
+    };
+    // candidates by first block id, in request order
+    std::unordered_map<int32_t, std::vector<int32_t>> by_first;
+    std::vector<int32_t> firsts;   // first ids in order of their first request
+    for (int32_t r = 0; r < R; ++r) {
+        group_of_req_out[r] = -1;
+        if (cap(r) < min_shared_blocks || row(r)[0] < 0) continue;
+        auto &v = by_first[row(r)[0]];
+        if (v.empty()) firsts.push_back(row(r)[0]);
+        v.push_back(r);
+    }
+    int32_t G = 0, nm = 0;
+    for (int32_t first : firsts) {
+        const std::vector<int32_t> &cand = by_first[first];
+        if (cand.size() < 2) continue;
+        const int32_t *ref = row(cand[0]);
+        // each member's shared run with the first candidate, within its cap
+        std::vector<int32_t> members;
+        int32_t shared = max_blocks;
+        for (int32_t r : cand) {
+            const int32_t c = cap(r), *rr = row(r);
+            int32_t k = 0;
+            while (k < c && rr[k] == ref[k] && rr[k] >= 0) ++k;
+            if (k < min_shared_blocks) continue;
+            members.push_back(r);
+            shared = std::min(shared, k);
+        }
+        if (members.size() < 2) continue;
+        for (int32_t r : members) {
+            group_of_req_out[r] = G;
+            member_req_out[nm++] = r;
+        }
+        group_blocks_out[G] = shared;
+        group_start_out[G + 1] = nm;
+        *max_group_blocks_out = std::max(*max_group_blocks_out, shared);
+        *max_group_members_out = std::max(*max_group_members_out, (int32_t)members.size());
+        ++G;
+    }
+    *num_groups_out = G;
+    return PKV_OK;
+}

@@ -35,7 +35,7 @@ EXPORTS = [
     "paged_attn_decode", "paged_attn_decode_noalloc", "paged_attn_decode_step", "pkv_trace_enable",
     "pkv_trace_read", "pkv_check_device_errors", "pkv_last_error", "pkv_prefix_cache_create",
     "pkv_prefix_cache_destroy", "pkv_prefix_cache_match", "pkv_prefix_cache_insert",
-    "pkv_prefix_cache_evict", "pkv_prefix_cache_size",
+    "pkv_prefix_cache_evict", "pkv_prefix_cache_size", "pkv_prefix_groups_build",
 ]
 
 
@@ -114,6 +114,7 @@ def load(path: str | None = None):
         "pkv_prefix_cache_insert": [V, P, i32, P, i32, P],
         "pkv_prefix_cache_evict": [V, i32, P, P],
         "pkv_prefix_cache_size": [V, P],
+        "pkv_prefix_groups_build": [P, i32, i32, P, i32, P, P, P, P, P, P, P],
         "pkv_trace_read": [V, P, i32, P],
     }
     for name, args in sig.items():
@@ -384,6 +385,28 @@ def pkv_prefix_cache_size(cache) -> int:
     n = np.zeros(1, np.int32)
     _check(load().pkv_prefix_cache_size(cache, _np_ptr(n)))
     return int(n[0])
+
+
+def pkv_prefix_groups_build(block_table, context_lens, min_shared_blocks: int = 1) -> dict:
+    """Prefix groups of a decode batch from its host block tables: a dict with
+    group_of_req, group_start, member_req, group_blocks (int32 numpy arrays),
+    num_groups, max_group_blocks, max_group_members."""
+    table = np.ascontiguousarray(block_table, np.int32)
+    ctx = np.ascontiguousarray(context_lens, np.int32)
+    R = table.shape[0]
+    gor = np.zeros(max(R, 1), np.int32)
+    gstart = np.zeros(R + 1, np.int32)
+    members = np.zeros(max(R, 1), np.int32)
+    gblocks = np.zeros(max(R, 1), np.int32)
+    cnt = np.zeros(3, np.int32)
+    _check(load().pkv_prefix_groups_build(
+        _np_ptr(table), table.shape[1], R, _np_ptr(ctx), int(min_shared_blocks), _np_ptr(gor),
+        _np_ptr(gstart), _np_ptr(members), _np_ptr(gblocks), _np_ptr(cnt[0:]), _np_ptr(cnt[1:]),
+        _np_ptr(cnt[2:])))
+    G = int(cnt[0])
+    return dict(group_of_req=gor[:R], group_start=gstart[:G + 1], member_req=members[:int(gstart[G])],
+                group_blocks=gblocks[:G], num_groups=G, max_group_blocks=int(cnt[1]),
+                max_group_members=int(cnt[2]))
 
 
 def pkv_trace_enable(pool, enable: bool = True):

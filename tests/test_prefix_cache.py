@@ -215,3 +215,93 @@ def test_matched_blocks_feed_decode():
         assert np.abs(lse[r].cpu().numpy() - l_ref[0]).max() <= 1e-3
     pkv.pkv_prefix_cache_destroy(cache)
     pkv.kv_pool_destroy(pool)
+
+
+# ---- prefix groups of a decode batch ----------------------------------------
+
+from oracle.prefix_cache import prefix_groups  # noqa: E402
+
+
+def test_groups_definition_hand_example():
+    pad = [-1] * 3
+    table = [[5, 6, 7, 8, 9] + pad,
+             [5, 6, 7, 20, 21] + pad,
+             [5, 6, 30, 31, 32] + pad,
+             [9, 10, 11, 12, 13] + pad,
+             [5, 6, 7, 8, 9] + pad]
+    L = [80, 80, 80, 80, 33]          # the last one: (33 - 1) // 16 = 2 shareable blocks
+    gor, groups = prefix_groups(table, L)
+    assert gor == [0, 0, 0, -1, 0] and groups == [([0, 1, 2, 4], 2)]
+    gor, groups = prefix_groups(table, L, min_shared_blocks=3)
+    assert gor == [0, 0, -1, -1, -1] and groups == [([0, 1], 3)]
+    gor, groups = prefix_groups(table, [16] * 5)       # one block each: nothing to share
+    assert gor == [-1] * 5 and groups == []
+
+
+def _check_groups(table, L, m):
+    got = pkv.pkv_prefix_groups_build(table, L, m)
+    gor, groups = prefix_groups(table.tolist(), list(L), m)
+    assert got["group_of_req"].tolist() == gor
+    assert got["num_groups"] == len(groups)
+    for g, (members, shared) in enumerate(groups):
+        a, b = got["group_start"][g], got["group_start"][g + 1]
+        assert got["member_req"][a:b].tolist() == members
+        assert int(got["group_blocks"][g]) == shared
+        for r in members:   # the shared blocks head every member's row, and leave it a private one
+            assert (table[r, :shared] == table[members[0], :shared]).all()
+            assert shared <= (L[r] - 1) // 16
+    if groups:
+        assert got["max_group_blocks"] == max(s for _, s in groups)
+        assert got["max_group_members"] == max(len(mm) for mm, _ in groups)
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2, 3])
+def test_groups_library_matches_definition(seed):
+    rng = np.random.default_rng(seed)
+    R, MB = 60, 40
+    runs = [rng.permutation(1000)[: int(rng.integers(1, 30))] for _ in range(5)]
+    table = np.full((R, MB), -1, np.int32)
+    L = np.zeros(R, np.int32)
+    nxt = 1000
+    for r in range(R):
+        k = int(rng.integers(0, 6))
+        head = runs[k][: int(rng.integers(0, len(runs[k]) + 1))] if k < 5 else np.zeros(0, np.int32)
+        nb = int(rng.integers(len(head) + 1, MB + 1))
+        own = np.arange(nxt, nxt + nb - len(head), dtype=np.int32)
+        nxt += nb - len(head)
+        table[r, :nb] = np.concatenate([head, own])
+        L[r] = 16 * (nb - 1) + int(rng.integers(1, 17))
+    for m in (1, 2, 5):
+        _check_groups(table, L, m)
+
+
+@pytest.mark.gpu
+def test_groups_from_tables_reproduce_the_workload_groups():
+    """On l8b_decode (scaled), groups derived from the block tables equal the
+    workload's own descriptor, and decode with them gives the same bits."""
+    import torch
+
+    from _lib import need_gpu
+    from paper_2605_11232_gb300 import batch as B
+    from paper_2605_11232_gb300.workloads import make_workload
+    need_gpu()
+    w = make_workload("l8b_decode", scale_requests=0.25)
+    b = B.build_batch(w, poison=True)
+    g = pkv.pkv_prefix_groups_build(b.table_host, w.context_lens)
+    assert g["num_groups"] == 1 and g["group_blocks"].tolist() == [w.prefix_lens[0] // 16]
+    assert (g["group_of_req"] == 0).all()
+    dev = {k: torch.from_numpy(g[k]).cuda() for k in ("group_start", "member_req", "group_blocks",
+                                                      "group_of_req")}
+    groups = pkv.make_prefix_groups(g["num_groups"], g["max_group_blocks"], g["max_group_members"], **dev)
+    B.run_write(b)
+    Rd = b.dec.stop - b.dec.start
+    outs = []
+    for grp in (b.groups, groups):
+        out = torch.empty((Rd, w.num_q_heads, w.head_dim), dtype=torch.bfloat16, device="cuda")
+        ws = torch.empty(pkv.paged_attn_decode_workspace_size(b.pool, Rd, w.num_q_heads, b.table.shape[1], grp),
+                         dtype=torch.uint8, device="cuda")
+        pkv.paged_attn_decode(b.pool, b.q, out, None, b.context_lens, b.table, w.scale, grp, ws)
+        outs.append(out.cpu())
+    assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
+    assert torch.equal(outs[0], outs[1])
+    b.close()
