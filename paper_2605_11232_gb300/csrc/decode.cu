@@ -393,35 +393,38 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(DecodeArgs a, Decod
         reinterpret_cast<const float2 *>(static_cast<const char *>(a.ws) + lay.off_ml);
     const int32_t *nparts =
         reinterpret_cast<const int32_t *>(static_cast<const char *>(a.ws) + lay.off_nparts);
-    // part counts written by the split pass: private pieces | prefix partials << 16
+    // The part counts written by the split pass (private pieces | prefix
+    // partials << 16) and, in the same round of loads, the (m, l) of every
+    // part slot: lane k holds slot k (prefix partials from 0, private pieces
+    // from prefix_parts); slots beyond the counts are masked once they are
+    // known (they may hold anything).
     const int32_t counts = nparts[item];
+    const int64_t head0 = (int64_t)r * lay.Hq + (int64_t)h * g;   // (request, q head) index of head 0
+    float2 mlv[G];
+#pragma unroll
+    for (int hd = 0; hd < G; ++hd) {
+        mlv[hd] = make_float2(-INFINITY, 0.f);
+        if (hd < g && lane < lay.parts_per_head) mlv[hd] = ml_part[(head0 + hd) * lay.parts_per_head + lane];
+    }
     const int n_priv = min(max(counts & 0xFFFF, 0), kMaxPrivateParts);
     const int n_pre = min((counts >> 16) & 0xFFFF, lay.prefix_parts);
     const int total = min(n_pre + n_priv, 32);
-    const int64_t head0 = (int64_t)r * lay.Hq + (int64_t)h * g;   // (request, q head) index of head 0
-    auto part_slot = [&](int hd, int k) {
-        return (head0 + hd) * lay.parts_per_head + (k < n_pre ? k : lay.prefix_parts + (k - n_pre));
-    };
-    // weights: lane k owns part k of every head
+    const bool live = lane < n_pre || (lane >= lay.prefix_parts && lane < lay.prefix_parts + n_priv);
+    // parts in merge order: the prefix partials, then the private pieces
+    auto part_lane = [&](int k) { return k < n_pre ? k : lay.prefix_parts + (k - n_pre); };
+    auto part_slot = [&](int hd, int k) { return (head0 + hd) * lay.parts_per_head + part_lane(k); };
+    // weights: the lane of a slot owns that slot's weight for every head
     float wk[G], mx[G], den[G];
 #pragma unroll
     for (int hd = 0; hd < G; ++hd) {
-        float2 v = make_float2(-INFINITY, 0.f);
-        if (hd < g && lane < total) v = ml_part[part_slot(hd, lane)];
-        mx[hd] = v.x;
-        wk[hd] = v.y;   // l for now
-    }
-#pragma unroll
-    for (int hd = 0; hd < G; ++hd) {
+        mx[hd] = (hd < g && live) ? mlv[hd].x : -INFINITY;
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) mx[hd] = fmaxf(mx[hd], __shfl_xor_sync(0xffffffffu, mx[hd], off));
     }
 #pragma unroll
     for (int hd = 0; hd < G; ++hd) {
-        float2 v = make_float2(-INFINITY, 0.f);
-        if (hd < g && lane < total) v = ml_part[part_slot(hd, lane)];
-        const float w = (hd < g && lane < total) ? fast_exp2(v.x - mx[hd]) : 0.f;
-        den[hd] = w * v.y;
+        const float w = (hd < g && live) ? fast_exp2(mlv[hd].x - mx[hd]) : 0.f;
+        den[hd] = (hd < g && live) ? w * mlv[hd].y : 0.f;
         wk[hd] = w;
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) den[hd] += __shfl_xor_sync(0xffffffffu, den[hd], off);
@@ -456,7 +459,7 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(DecodeArgs a, Decod
         for (int u = 0; u < KR; ++u)
 #pragma unroll
             for (int hd = 0; hd < G; ++hd) {
-                const float w = __shfl_sync(0xffffffffu, wk[hd], (k0 + u) & 31);
+                const float w = __shfl_sync(0xffffffffu, wk[hd], k0 + u < total ? part_lane(k0 + u) : 0);
 #pragma unroll
                 for (int e = 0; e < E; ++e) acc[hd][e] += w * v[u][hd][e];
             }
