@@ -415,11 +415,19 @@ int paged_attn_decode_workspace_size(pkv_pool_t pool, int32_t num_requests, int3
     return ok();
 }
 
-int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
-                      const int32_t *context_lens, const int32_t *block_table, int32_t max_blocks,
-                      int32_t num_requests, int32_t num_q_heads, float scale,
-                      const pkv_prefix_groups *groups, void *workspace, size_t workspace_bytes,
-                      pkv_stream_t stream) {
+}  // extern "C"
+
+namespace {
+
+// Every host-side check of paged_attn_decode, then its layout and kernel
+// arguments (and the pool's TMA descriptors when the prefix pass runs);
+// nothing is enqueued.  *empty: no request, nothing to launch.
+int prepare_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
+                   const int32_t *context_lens, const int32_t *block_table, int32_t max_blocks,
+                   int32_t num_requests, int32_t num_q_heads, float scale,
+                   const pkv_prefix_groups *groups, void *workspace, size_t workspace_bytes,
+                   pkv::DecodeLayout *L_out, pkv::DecodeArgs *a_out, bool *empty) {
+    *empty = true;
     int rc = check_kernel_pool(pool);
     if (rc != PKV_OK) return rc;
     const pkv_pool_desc &d = pool->desc;
@@ -430,7 +438,8 @@ int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
     if (g > 8) return fail(PKV_ERR_UNSUPPORTED, "decode supports up to 8 q heads per kv head");
     if (num_requests > 16384) return fail(PKV_ERR_UNSUPPORTED, "decode supports up to 16384 requests");
     if (!(scale > 0.f) || !std::isfinite(scale)) return fail(PKV_ERR_INVALID_ARG, "bad scale");
-    if (num_requests == 0) return ok();
+    *empty = num_requests == 0;
+    if (*empty) return ok();
     if (!q || !out || !context_lens || !block_table) return fail(PKV_ERR_INVALID_ARG, "NULL buffer");
     if (!aligned16(q) || !aligned16(out)) return fail(PKV_ERR_INVALID_ARG, "misaligned q/out");
     int32_t G = 0, mgb = 0, mgm = 0;
@@ -444,7 +453,8 @@ int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
         if (mgb > max_blocks) return fail(PKV_ERR_INVALID_ARG, "max_group_blocks exceeds the table width");
         if ((int64_t)G * d.num_kv_heads > INT32_MAX) return fail(PKV_ERR_UNSUPPORTED, "too many groups");
     }
-    pkv::DecodeLayout L = pkv::decode_layout(num_requests, num_q_heads, d.num_kv_heads, d.head_dim,
+    pkv::DecodeLayout &L = *L_out;
+    L = pkv::decode_layout(num_requests, num_q_heads, d.num_kv_heads, d.head_dim,
                                              max_blocks, G, mgb, mgm, pool->num_sms);
     if (!workspace || workspace_bytes < L.total)
         return fail(PKV_ERR_WORKSPACE, "workspace of %zu bytes needed", L.total);
@@ -452,7 +462,8 @@ int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
         return fail(PKV_ERR_WORKSPACE, "workspace must be 256-byte aligned");
     if ((rc = set_device(pool)) != PKV_OK) return rc;
     if (L.prefix_parts > 0 && (rc = build_tmaps(pool)) != PKV_OK) return rc;
-    pkv::DecodeArgs a{};
+    pkv::DecodeArgs &a = *a_out;
+    a = pkv::DecodeArgs{};
     a.q = q; a.out = out; a.lse = lse;
     a.context_lens = context_lens; a.block_table = block_table; a.max_blocks = max_blocks;
     a.k_cache = pool->k_cache; a.v_cache = pool->v_cache;
@@ -468,7 +479,25 @@ int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
     a.sched = pool->d_err + 1;
     a.tmap_k = &pool->tmap_k;
     a.tmap_v = &pool->tmap_v;
-    cudaError_t e = pkv::launch_decode(L, a, pool->num_sms, d.num_blocks,
+    return ok();
+}
+
+}  // namespace
+
+extern "C" {
+
+int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
+                      const int32_t *context_lens, const int32_t *block_table, int32_t max_blocks,
+                      int32_t num_requests, int32_t num_q_heads, float scale,
+                      const pkv_prefix_groups *groups, void *workspace, size_t workspace_bytes,
+                      pkv_stream_t stream) {
+    pkv::DecodeLayout L{};
+    pkv::DecodeArgs a{};
+    bool empty = true;
+    const int rc = prepare_decode(pool, q, out, lse, context_lens, block_table, max_blocks, num_requests,
+                                  num_q_heads, scale, groups, workspace, workspace_bytes, &L, &a, &empty);
+    if (rc != PKV_OK || empty) return rc;
+    cudaError_t e = pkv::launch_decode(L, a, pool->num_sms, pool->desc.num_blocks,
                                        static_cast<cudaStream_t>(stream), pool->tracer);
     if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode launch");
     return ok();
@@ -501,6 +530,16 @@ int paged_attn_decode_step(pkv_pool_t pool, const void *host_in, void *dev_in,
         if (g.off % 16 != 0 || g.off > layout->bytes || g.len > layout->bytes - g.off)
             return fail(PKV_ERR_INVALID_ARG, "step layout: region at %zu (%zu bytes) misaligned or "
                         "outside the %zu-byte buffer", g.off, g.len, layout->bytes);
+    // every argument check before anything is enqueued
+    const char *din = static_cast<const char *>(dev_in);
+    pkv::DecodeLayout L{};
+    pkv::DecodeArgs a{};
+    bool empty = true;
+    rc = prepare_decode(pool, din + layout->q, out, lse,
+                        reinterpret_cast<const int32_t *>(din + layout->context_lens), block_table,
+                        max_blocks, num_requests, num_q_heads, scale, groups, workspace, workspace_bytes,
+                        &L, &a, &empty);
+    if (rc != PKV_OK) return rc;
     if ((rc = set_device(pool)) != PKV_OK) return rc;
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     cudaError_t e = cudaMemcpyAsync(dev_in, host_in, layout->bytes, cudaMemcpyHostToDevice, st);
@@ -509,16 +548,14 @@ int paged_attn_decode_step(pkv_pool_t pool, const void *host_in, void *dev_in,
         e = cudaStreamWaitEvent(st, static_cast<cudaEvent_t>(wait_event), 0);
         if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode_step wait_event");
     }
-    const char *din = static_cast<const char *>(dev_in);
     rc = kv_cache_write(pool, din + layout->k_new, din + layout->v_new,
                         reinterpret_cast<const int64_t *>(din + layout->slot_mapping), num_new_tokens,
                         stream);
     if (rc != PKV_OK) return rc;
-    rc = paged_attn_decode(pool, din + layout->q, out, lse,
-                           reinterpret_cast<const int32_t *>(din + layout->context_lens), block_table,
-                           max_blocks, num_requests, num_q_heads, scale, groups, workspace,
-                           workspace_bytes, stream);
-    if (rc != PKV_OK) return rc;
+    if (!empty) {
+        e = pkv::launch_decode(L, a, pool->num_sms, d.num_blocks, st, pool->tracer);
+        if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode_step launch");
+    }
     if (done_event) {
         e = cudaEventRecord(static_cast<cudaEvent_t>(done_event), st);
         if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode_step done_event");

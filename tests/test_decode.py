@@ -249,7 +249,10 @@ def test_decode_step_from_host_buffers_bit_exact(groups):
         torch.cuda.synchronize()
         assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
         assert torch.equal(host_out, ref.cpu()) and torch.equal(host_lse, ref_lse.cpu())
-    # a misaligned region is refused before anything is enqueued
+    # a misaligned region, or a decode argument error, is refused before
+    # anything is enqueued: the device input buffer keeps its contents
+    dev.fill_(0xAB)
+    torch.cuda.synchronize()
     bad = pkv.StepLayout(q=layout.q, k_new=layout.k_new + 8, v_new=layout.v_new,
                          slot_mapping=layout.slot_mapping, context_lens=layout.context_lens,
                          bytes=layout.bytes)
@@ -257,6 +260,12 @@ def test_decode_step_from_host_buffers_bit_exact(groups):
         pkv.paged_attn_decode_step(b.pool, hosts[0], dev, bad, w.num_new_tokens, b.table[b.dec],
                                    w.num_q_heads, w.scale, None, ws, out)
     assert e.value.code == pkv.PKV_ERR_INVALID_ARG
+    with pytest.raises(pkv.PkvError) as e:
+        pkv.paged_attn_decode_step(b.pool, hosts[0], dev, layout, w.num_new_tokens, b.table[b.dec],
+                                   w.num_q_heads + 1, w.scale, None, ws, out)
+    assert e.value.code == pkv.PKV_ERR_INVALID_ARG
+    torch.cuda.synchronize()
+    assert bool((dev == 0xAB).all())
     b.close()
 
 
