@@ -200,3 +200,18 @@ def test_speculative_verify_chain_drafts():
     out, lse = run_prefill(b)
     compare(b, out, lse, range(R))
     b.close()
+
+
+def test_prefill_longest_item_and_empty_request():
+    """A work item at the longest key range one item may span (32,760 cached
+    tokens + 4 queries: 2048 blocks), beside a request with no new tokens (it
+    reads and writes nothing) and a short one: every row of the two against
+    the oracle."""
+    need_gpu()
+    w = make_workload("custom", seed=3, custom=dict(
+        Hq=8, Hkv=1, d=128, prefix_lens=[], group=[-1] * 3, cached=[32760, 10, 500],
+        new=[4, 0, 7], decode=[False] * 3))
+    b = B.build_batch(w, poison=True)
+    out, lse = run_prefill(b)
+    compare(b, out, lse, [0, 2])
+    b.close()
