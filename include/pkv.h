@@ -15,8 +15,9 @@
  * the cache write (kv_cache_write), suffix prefill (paged_attn_prefill),
  * decode (paged_attn_decode; without a caller workspace:
  * paged_attn_decode_noalloc; one host-driven step with its copies:
- * paged_attn_decode_step), per-kernel tracing (pkv_trace_*) and device error
- * reporting (pkv_check_device_errors).
+ * paged_attn_decode_step), per-kernel tracing (pkv_trace_*), device error
+ * reporting (pkv_check_device_errors) and a test aid for it
+ * (pkv_selftest_wait_timeout).
  *
  * Conventions for every call
  *  - All device buffers are owned by the caller.  The library keeps host
@@ -361,6 +362,16 @@ int paged_attn_decode_noalloc(pkv_pool_t pool, const void *q, void *out, float *
                               const int32_t *context_lens, const int32_t *block_table,
                               int32_t max_blocks, int32_t num_requests, int32_t num_q_heads,
                               float scale, const pkv_prefix_groups *groups, pkv_stream_t stream);
+
+/* ---- test aid ------------------------------------------------------------ */
+
+/* Make one bounded device wait run out: a single thread waits, with the same
+ * bounded mbarrier wait as the kernels, on a phase that nothing completes,
+ * for limit_us microseconds (0 .. 1e6), then latches DEVICE_TIMEOUT into the
+ * pool's error word and returns (no copy, MMA or tensor memory involved).
+ * pkv_check_device_errors then reports PKV_ERR_DEVICE_TIMEOUT, and the
+ * context stays usable.  Errors: INVALID_ARG, CUDA. */
+int pkv_selftest_wait_timeout(pkv_pool_t pool, int32_t limit_us, pkv_stream_t stream);
 
 /* ---- tracing -------------------------------------------------------------- */
 

@@ -179,6 +179,14 @@ int set_last_error(int code, const char *msg) {
     g_last_error = msg ? msg : "";
     return code;
 }
+
+int pool_device_error_word(pkv_pool_t pool, int **err) {
+    int rc = check_kernel_pool(pool);
+    if (rc != PKV_OK) return rc;
+    if ((rc = set_device(pool)) != PKV_OK) return rc;
+    *err = pool->d_err;
+    return PKV_OK;
+}
 }  // namespace pkv
 
 extern "C" {

@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+struct pkv_pool;   // the pool handle's struct (include/pkv.h: pkv_pool_t)
+
 namespace pkv {
 
 // Kernels the library launches (names reported by pkv_trace_read).
@@ -50,6 +52,10 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 
 // Set the thread's pkv_last_error() message; returns code.
 int set_last_error(int code, const char *msg);
+
+// The pool's device error word, after checking that the pool has device
+// caches and making its device current; PKV_OK or an error code.
+int pool_device_error_word(::pkv_pool *pool, int **err);
 
 // Device error word values (a kernel latches the first one with atomicCAS).
 enum : int {

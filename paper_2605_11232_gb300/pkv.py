@@ -36,6 +36,7 @@ EXPORTS = [
     "pkv_trace_read", "pkv_check_device_errors", "pkv_last_error", "pkv_prefix_cache_create",
     "pkv_prefix_cache_destroy", "pkv_prefix_cache_match", "pkv_prefix_cache_insert",
     "pkv_prefix_cache_evict", "pkv_prefix_cache_size", "pkv_prefix_groups_build",
+    "pkv_selftest_wait_timeout",
 ]
 
 
@@ -115,6 +116,7 @@ def load(path: str | None = None):
         "pkv_prefix_cache_evict": [V, i32, P, P],
         "pkv_prefix_cache_size": [V, P],
         "pkv_prefix_groups_build": [P, i32, i32, P, i32, P, P, P, P, P, P, P],
+        "pkv_selftest_wait_timeout": [V, i32, V],
         "pkv_trace_read": [V, P, i32, P],
     }
     for name, args in sig.items():
@@ -407,6 +409,11 @@ def pkv_prefix_groups_build(block_table, context_lens, min_shared_blocks: int = 
     return dict(group_of_req=gor[:R], group_start=gstart[:G + 1], member_req=members[:int(gstart[G])],
                 group_blocks=gblocks[:G], num_groups=G, max_group_blocks=int(cnt[1]),
                 max_group_members=int(cnt[2]))
+
+
+def pkv_selftest_wait_timeout(pool, limit_us: int = 1000, stream=None):
+    """Test aid: one bounded device wait runs out and latches DEVICE_TIMEOUT."""
+    _check(load().pkv_selftest_wait_timeout(pool, int(limit_us), _stream(stream)))
 
 
 def pkv_trace_enable(pool, enable: bool = True):
