@@ -84,6 +84,14 @@ def decode_bytes(w, req):
     return rows * kv_row_bytes(w) + 2 * nq * w.num_q_heads * w.head_dim * 2
 
 
+def decode_logical_bytes(w, req):
+    """Every decode request's K/V rows (a shared prefix counted once per
+    request, as a cache without sharing would read it) + Q + O."""
+    rows = sum(int(w.context_lens[r]) for r in range(req.start, req.stop))
+    nq = req.stop - req.start
+    return rows * kv_row_bytes(w) + 2 * nq * w.num_q_heads * w.head_dim * 2
+
+
 def write_bytes(w, ntok):
     return 2 * ntok * kv_row_bytes(w)                # read new K/V + write into the pool
 
@@ -318,6 +326,7 @@ def measure_workload(name, steps, warmup, use_groups=True, e2e_steps=0):
     res = dict(name=name, w=w, step_ms=step_ms, warm_ms=warm_ms, trace=trace, groups=groups_ok,
                kernel_bytes=kb,
                dec_bytes=decode_bytes(w, b.dec) if Rd else 0,
+               dec_logical=decode_logical_bytes(w, b.dec) if Rd else 0,
                wr_bytes=write_bytes(w, w.num_new_tokens),
                pre_flops=prefill_flops(w, b.pre) if Rp else 0, Rd=Rd, Rp=Rp)
 
@@ -391,12 +400,17 @@ def summarize(res, peaks):
             # (per-launch CUDA events), not over a step that also runs prefill
             dec_us = sum(1e3 * t / n for k, (n, t) in res["trace"].items() if k.startswith("decode_"))
             gbs = res["dec_bytes"] / (dec_us * 1e-6) / 1e9 if dec_us > 0 else float("nan")
+            logical = res.get("dec_logical", 0) / (dec_us * 1e-6) / 1e9 if dec_us > 0 else float("nan")
             basis = "decode kernels' CUDA-event time"
         else:
             gbs = (res["dec_bytes"] + res["wr_bytes"]) / (ms * 1e-3) / 1e9
+            logical = (res.get("dec_logical", 0) + res["wr_bytes"]) / (ms * 1e-3) / 1e9
             basis = "whole step (cache write + decode)"
         out.update(decode_hbm_gbs=gbs, decode_frac_of_measured_hbm=gbs / hbm,
-                   decode_frac_of_8tbs=gbs / 8000.0, decode_basis=basis, prefix_pass=res["groups"])
+                   decode_frac_of_8tbs=gbs / 8000.0, decode_basis=basis, prefix_pass=res["groups"],
+                   decode_logical_gbs=logical,
+                   decode_logical_note="logical: every request's K/V rows, a shared prefix counted "
+                                       "once per request (what a cache without sharing reads)")
         if not res["Rp"]:
             out["decode_hbm_gbs_warm_l2"] = (res["dec_bytes"] + res["wr_bytes"]) / (
                 statistics.mean(res["warm_ms"]) * 1e-3) / 1e9
