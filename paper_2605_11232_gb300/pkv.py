@@ -3,6 +3,12 @@
 Every function here forwards to the C entry point of the same name.  Device
 buffers are torch CUDA tensors owned by the caller; host arrays are numpy.
 There is no fallback: if the library cannot be loaded, every call raises.
+
+The C entry points take bare device pointers, so they cannot see a tensor of
+the wrong dtype or with too few rows.  The wrappers of the kernel calls
+therefore check each tensor's dtype and shape against the layout the entry
+point reads (ValueError) before any pointer is taken: a mismatch that would
+make a kernel read or write past a buffer is refused on the host.
 """
 
 from __future__ import annotations
@@ -149,6 +155,68 @@ def _dptr(t):
     return ctypes.c_void_p(t.data_ptr())
 
 
+# (num_blocks, num_kv_heads, head_dim) of every pool this module created
+_POOL_GEOMETRY: dict = {}
+
+
+def _need(cond, msg):
+    if not cond:
+        raise ValueError(msg)
+
+
+def _pool_geometry(pool):
+    key = pool.value if isinstance(pool, ctypes.c_void_p) else pool
+    return _POOL_GEOMETRY.get(key)
+
+
+def _check_tensor(name, t, dtype, ndim):
+    _need(t is not None, f"{name} is required")
+    _need(t.dtype == dtype, f"{name} must be {dtype}, got {t.dtype}")
+    _need(t.dim() == ndim, f"{name} must have {ndim} dimensions, got shape {tuple(t.shape)}")
+
+
+def _check_cache_write_args(pool, k_new, v_new, slot_mapping):
+    """k_new, v_new bf16 [>= T][Hkv][d]; slot_mapping int64 [T]."""
+    import torch
+    _check_tensor("slot_mapping", slot_mapping, torch.int64, 1)
+    T = slot_mapping.shape[0]
+    geo = _pool_geometry(pool)
+    for name, t in (("k_new", k_new), ("v_new", v_new)):
+        _check_tensor(name, t, torch.bfloat16, 3)
+        _need(t.shape[0] >= T, f"{name} has {t.shape[0]} rows for {T} slots")
+        if geo is not None:
+            _need(tuple(t.shape[1:]) == geo[1:],
+                  f"{name} rows must be [num_kv_heads][head_dim] = {list(geo[1:])}, "
+                  f"got {list(t.shape[1:])}")
+
+
+def _check_attn_args(pool, q, out, lse, context_lens, block_table, min_q_rows):
+    """q bf16 [>= min_q_rows][Hq][d] with d the pool's head dim and Hq a
+    multiple of its kv heads; out bf16 with q's row layout; lse fp32 [.][Hq]
+    or None; context_lens int32 [R]; block_table int32 [>= R][max_blocks]."""
+    import torch
+    _check_tensor("context_lens", context_lens, torch.int32, 1)
+    R = context_lens.shape[0]
+    _check_tensor("block_table", block_table, torch.int32, 2)
+    _need(block_table.shape[0] >= R, f"block_table has {block_table.shape[0]} rows for {R} requests")
+    _need(block_table.shape[1] >= 1, "block_table needs at least one column")
+    _check_tensor("q", q, torch.bfloat16, 3)
+    _need(q.shape[0] >= min_q_rows, f"q has {q.shape[0]} rows, {min_q_rows} needed")
+    geo = _pool_geometry(pool)
+    if geo is not None:
+        _need(q.shape[2] == geo[2], f"q head dim {q.shape[2]} != the pool's {geo[2]}")
+        _need(q.shape[1] % geo[1] == 0,
+              f"{q.shape[1]} query heads are not a multiple of the pool's {geo[1]} kv heads")
+    _check_tensor("out", out, torch.bfloat16, 3)
+    _need(tuple(out.shape[1:]) == tuple(q.shape[1:]),
+          f"out rows must be {list(q.shape[1:])}, got {list(out.shape[1:])}")
+    _need(out.shape[0] >= min_q_rows, f"out has {out.shape[0]} rows, {min_q_rows} needed")
+    if lse is not None:
+        _check_tensor("lse", lse, torch.float32, 2)
+        _need(lse.shape[1] == q.shape[1], f"lse must have {q.shape[1]} columns, got {lse.shape[1]}")
+        _need(lse.shape[0] >= min_q_rows, f"lse has {lse.shape[0]} rows, {min_q_rows} needed")
+
+
 def _stream(stream):
     if stream is None:
         import torch
@@ -164,14 +232,22 @@ def kv_pool_create(num_blocks: int, num_kv_heads: int, head_dim: int, k_cache=No
                    v_cache=None, placement_seed: int = 0, block_size: int = 16):
     desc = PoolDesc(num_blocks, block_size, num_kv_heads, head_dim, PKV_DTYPE_BF16, 0,
                     placement_seed & (2**64 - 1))
+    if k_cache is not None or v_cache is not None:
+        import torch
+        shape = (num_blocks, num_kv_heads, block_size, head_dim)
+        for name, t in (("k_cache", k_cache), ("v_cache", v_cache)):
+            _check_tensor(name, t, torch.bfloat16, 4)
+            _need(tuple(t.shape) == shape, f"{name} must have shape {list(shape)}, got {list(t.shape)}")
     h = ctypes.c_void_p()
     _check(load().kv_pool_create(ctypes.byref(desc), _dptr(k_cache), _dptr(v_cache),
                                  ctypes.byref(h)))
+    _POOL_GEOMETRY[h.value] = (int(num_blocks), int(num_kv_heads), int(head_dim))
     return h
 
 
 def kv_pool_destroy(pool):
     _check(load().kv_pool_destroy(pool))
+    _POOL_GEOMETRY.pop(pool.value if isinstance(pool, ctypes.c_void_p) else pool, None)
 
 
 def kv_pool_alloc(pool, n: int) -> np.ndarray:
@@ -232,12 +308,21 @@ def kv_slot_mapping(pool, block_table: np.ndarray, context_lens, new_lens,
 # ---- a3-a7: kernels ---------------------------------------------------------
 
 def kv_cache_write(pool, k_new, v_new, slot_mapping, stream=None):
+    _check_cache_write_args(pool, k_new, v_new, slot_mapping)
     _check(load().kv_cache_write(pool, _dptr(k_new), _dptr(v_new), _dptr(slot_mapping),
                                  int(slot_mapping.shape[0]), _stream(stream)))
 
 
 def paged_attn_prefill(pool, q, out, lse, cu_seqlens_q, context_lens, block_table,
                        max_seqlen_q: int, scale: float, stream=None):
+    import torch
+    _check_attn_args(pool, q, out, lse, context_lens, block_table, 0)
+    _need(tuple(out.shape) == tuple(q.shape), f"out must have q's shape {list(q.shape)}")
+    if lse is not None:
+        _need(lse.shape[0] == q.shape[0], f"lse must have {q.shape[0]} rows")
+    _check_tensor("cu_seqlens_q", cu_seqlens_q, torch.int32, 1)
+    _need(cu_seqlens_q.shape[0] == context_lens.shape[0] + 1,
+          f"cu_seqlens_q must have {context_lens.shape[0] + 1} entries")
     _check(load().paged_attn_prefill(
         pool, _dptr(q), _dptr(out), _dptr(lse), _dptr(cu_seqlens_q), _dptr(context_lens),
         _dptr(block_table), int(block_table.shape[1]), int(context_lens.shape[0]),
@@ -246,6 +331,12 @@ def paged_attn_prefill(pool, q, out, lse, cu_seqlens_q, context_lens, block_tabl
 
 def make_prefix_groups(num_groups=0, max_group_blocks=0, max_group_members=0, group_start=None,
                        member_req=None, group_blocks=None, group_of_req=None):
+    import torch
+    for name, t, n in (("group_start", group_start, num_groups + 1), ("member_req", member_req, 0),
+                       ("group_blocks", group_blocks, num_groups), ("group_of_req", group_of_req, 0)):
+        if t is not None or num_groups > 0:
+            _check_tensor(name, t, torch.int32, 1)
+            _need(t.shape[0] >= n, f"{name} has {t.shape[0]} entries, {n} needed")
     return PrefixGroups(int(num_groups), int(max_group_blocks), int(max_group_members), 0,
                         _dptr(group_start), _dptr(member_req), _dptr(group_blocks),
                         _dptr(group_of_req))
@@ -262,6 +353,7 @@ def paged_attn_decode_workspace_size(pool, num_requests: int, num_q_heads: int,
 
 def paged_attn_decode(pool, q, out, lse, context_lens, block_table, scale: float, groups,
                       workspace, stream=None):
+    _check_attn_args(pool, q, out, lse, context_lens, block_table, int(context_lens.shape[0]))
     _check(load().paged_attn_decode(
         pool, _dptr(q), _dptr(out), _dptr(lse), _dptr(context_lens), _dptr(block_table),
         int(block_table.shape[1]), int(context_lens.shape[0]), int(q.shape[1]), float(scale),
@@ -273,6 +365,7 @@ def paged_attn_decode(pool, q, out, lse, context_lens, block_table, scale: float
 def paged_attn_decode_noalloc(pool, q, out, lse, context_lens, block_table, scale: float,
                               groups, stream=None):
     """paged_attn_decode with the library's static scratch (no workspace)."""
+    _check_attn_args(pool, q, out, lse, context_lens, block_table, int(context_lens.shape[0]))
     _check(load().paged_attn_decode_noalloc(
         pool, _dptr(q), _dptr(out), _dptr(lse), _dptr(context_lens), _dptr(block_table),
         int(block_table.shape[1]), int(context_lens.shape[0]), int(q.shape[1]), float(scale),
