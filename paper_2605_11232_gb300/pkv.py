@@ -390,8 +390,41 @@ def _event(ev):
     return ctypes.c_void_p(ev.cuda_event)
 
 
+def _check_step_args(pool, host_in, dev_in, layout, block_table, num_q_heads, out, lse,
+                     host_out, host_lse):
+    """Both step buffers hold layout.bytes (the H2D copy moves that many);
+    out bf16 [>= R][num_q_heads][d] and lse fp32 [>= R][num_q_heads] as the
+    kernels write them; host_out / host_lse the same shape and dtype as the
+    device tensors they receive."""
+    import torch
+    for name, t in (("host_in", host_in), ("dev_in", dev_in)):
+        _need(t is not None, f"{name} is required")
+        nbytes = t.numel() * t.element_size()
+        _need(nbytes >= layout.bytes, f"{name} holds {nbytes} bytes, the layout needs {layout.bytes}")
+    _check_tensor("block_table", block_table, torch.int32, 2)
+    R = block_table.shape[0]
+    _check_tensor("out", out, torch.bfloat16, 3)
+    _need(out.shape[0] >= R and out.shape[1] == num_q_heads,
+          f"out must be [>= {R}][{num_q_heads}][head_dim], got {list(out.shape)}")
+    geo = _pool_geometry(pool)
+    if geo is not None:
+        _need(out.shape[2] == geo[2], f"out head dim {out.shape[2]} != the pool's {geo[2]}")
+    if lse is not None:
+        _check_tensor("lse", lse, torch.float32, 2)
+        _need(lse.shape[0] >= R and lse.shape[1] == num_q_heads,
+              f"lse must be [>= {R}][{num_q_heads}], got {list(lse.shape)}")
+    for name, h, d in (("host_out", host_out, out), ("host_lse", host_lse, lse)):
+        if h is not None:
+            _need(d is not None, f"{name} needs its device tensor")
+            _need(h.dtype == d.dtype and tuple(h.shape) == tuple(d.shape),
+                  f"{name} must match its device tensor ({d.dtype} {list(d.shape)}), "
+                  f"got {h.dtype} {list(h.shape)}")
+
+
 def _step_args(pool, host_in, dev_in, layout, num_new_tokens, block_table, num_q_heads, scale,
                groups, workspace, out, lse, host_out, host_lse, wait_event, done_event, stream):
+    _check_step_args(pool, host_in, dev_in, layout, block_table, num_q_heads, out, lse, host_out,
+                     host_lse)
     return (pool, _hptr(host_in), _dptr(dev_in), ctypes.byref(layout), int(num_new_tokens),
             _dptr(block_table), int(block_table.shape[1]), int(block_table.shape[0]),
             int(num_q_heads), float(scale), ctypes.byref(groups) if groups is not None else None,

@@ -134,3 +134,36 @@ def test_prefix_group_checks():
     reaches_device_check(mk, G, 5, 2, gs, mr, gb, gor)
     # no groups: an empty descriptor needs no tensors
     assert mk().num_groups == 0
+
+
+def test_decode_step_checks(pool):
+    R, T = 4, 4
+    layout = pkv.StepLayout(q=0, k_new=1024, v_new=2048, slot_mapping=3072, context_lens=3328,
+                            bytes=3456)
+    host = torch.zeros(layout.bytes, dtype=torch.uint8)
+    dev = torch.zeros(layout.bytes, dtype=torch.uint8)
+    table = torch.zeros((R, 3), dtype=torch.int32)
+    out = torch.zeros((R, HQ, D), dtype=BF)
+    lse = torch.zeros((R, HQ), dtype=torch.float32)
+    ws = torch.zeros(1024, dtype=torch.uint8)
+
+    def call(**kw):
+        a = dict(host_in=host, dev_in=dev, block_table=table, num_q_heads=HQ, out=out, lse=lse,
+                 host_out=None, host_lse=None)
+        a.update(kw)
+        return pkv.paged_attn_decode_step(pool, a["host_in"], a["dev_in"], layout, T, a["block_table"],
+                                          a["num_q_heads"], 0.125, None, ws, a["out"], a["lse"],
+                                          a["host_out"], a["host_lse"])
+
+    refused("host_in holds 3440 bytes, the layout needs 3456", lambda: call(host_in=host[:-16]))
+    refused("dev_in holds 3440 bytes", lambda: call(dev_in=dev[:-16]))
+    refused("block_table must be torch.int32", lambda: call(block_table=table.long()))
+    refused(re.escape("out must be [>= 4][8][head_dim]"), lambda: call(out=out[:3]))
+    refused(re.escape("out must be [>= 4][9][head_dim]"), lambda: call(num_q_heads=HQ + 1))
+    refused("out head dim 128 != the pool's 64", lambda: call(out=torch.zeros((R, HQ, 128), dtype=BF)))
+    refused(re.escape("lse must be [>= 4][8]"), lambda: call(lse=lse[:, :4].contiguous()))
+    refused("host_out must match", lambda: call(host_out=torch.zeros((R - 1, HQ, D), dtype=BF)))
+    refused("host_lse needs its device tensor",
+            lambda: call(lse=None, host_lse=torch.zeros((R, HQ), dtype=torch.float32)))
+    # a host buffer passes the checks and stops at the device check of dev_in
+    reaches_device_check(lambda: call(host_out=torch.zeros_like(out), host_lse=torch.zeros_like(lse)))

@@ -260,9 +260,11 @@ def test_decode_step_from_host_buffers_bit_exact(groups):
         pkv.paged_attn_decode_step(b.pool, hosts[0], dev, bad, w.num_new_tokens, b.table[b.dec],
                                    w.num_q_heads, w.scale, None, ws, out)
     assert e.value.code == pkv.PKV_ERR_INVALID_ARG
+    out_more_heads = torch.empty((R, w.num_q_heads + 1, w.head_dim), dtype=torch.bfloat16,
+                                 device="cuda")
     with pytest.raises(pkv.PkvError) as e:
         pkv.paged_attn_decode_step(b.pool, hosts[0], dev, layout, w.num_new_tokens, b.table[b.dec],
-                                   w.num_q_heads + 1, w.scale, None, ws, out)
+                                   w.num_q_heads + 1, w.scale, None, ws, out_more_heads)
     assert e.value.code == pkv.PKV_ERR_INVALID_ARG
     torch.cuda.synchronize()
     assert bool((dev == 0xAB).all())
