@@ -93,7 +93,12 @@ typedef struct {
  * entries are the same physical blocks for every member, hold full 16-token
  * blocks of the shared prefix, and are never written.  With groups, decode
  * reads each shared block once per group and kv head instead of once per
- * request.  All arrays are device arrays. */
+ * request.  All arrays are device arrays.  The two host bounds size the
+ * workspace and the prefix pass's grid; the device arrays are not read on the
+ * host, so a group with more blocks or members than the bounds is not
+ * detected: the kernels stay inside the workspace and the tables, but the
+ * blocks or members past a bound are left out of that request's attention.
+ * pkv_prefix_groups_build returns exact bounds. */
 typedef struct {
     int32_t num_groups;        /* G >= 0; 0 means no sharing information         */
     int32_t max_group_blocks;  /* host upper bound on group_blocks[g]            */

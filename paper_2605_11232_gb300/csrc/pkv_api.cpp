@@ -331,7 +331,7 @@ int kv_slot_mapping(pkv_pool_t pool, const int32_t *block_table, int32_t max_blo
     int64_t t = 0;
     for (int32_t r = 0; r < num_requests; ++r) {
         const int32_t L = context_lens[r], n = new_lens[r];
-        if (n < 0 || L < n || (L + 15) / 16 > max_blocks)
+        if (n < 0 || L < n || ((int64_t)L + 15) / 16 > max_blocks)
             return fail(PKV_ERR_INVALID_ARG, "request %d: context %d, new %d, table width %d", r, L,
                         n, max_blocks);
         for (int32_t i = 0; i < n; ++i) {

@@ -101,6 +101,19 @@ def test_slot_mapping_matches_oracle_and_rejects_shared_writes(pool):
     assert np.array_equal(got2, oracle.slot_mapping(table, ctx, [1, 10, 60], 16))
 
 
+def test_slot_mapping_rejects_contexts_wider_than_the_table():
+    """A context longer than 16 x the table width is refused before any table
+    entry is read, up to the largest int32 length (no overflow in the width
+    test)."""
+    built_lib()
+    table = np.zeros((1, 4), np.int32)
+    for L in (65, 2**31 - 16, 2**31 - 8, 2**31 - 1):
+        with pytest.raises(pkv.PkvError) as e:
+            pkv.kv_slot_mapping(None, table, [L], [1])
+        assert e.value.code == pkv.PKV_ERR_INVALID_ARG
+    assert list(pkv.kv_slot_mapping(None, table, [64], [1])) == [63]
+
+
 def test_kernel_calls_need_device_caches(pool):
     with pytest.raises(pkv.PkvError) as e:
         pkv._check(pkv.load().kv_cache_write(pool, None, None, None, 1, None))
