@@ -106,7 +106,7 @@ def test_slot_mapping_rejects_contexts_wider_than_the_table():
     entry is read, up to the largest int32 length (no overflow in the width
     test)."""
     built_lib()
-    table = np.zeros((1, 4), np.int32)
+    table = np.arange(4, dtype=np.int32)[None, :]
     for L in (65, 2**31 - 16, 2**31 - 8, 2**31 - 1):
         with pytest.raises(pkv.PkvError) as e:
             pkv.kv_slot_mapping(None, table, [L], [1])
