@@ -160,8 +160,10 @@ _POOL_GEOMETRY: dict = {}
 
 
 def _need(cond, msg):
+    """Raise ValueError unless cond; msg is a string or a callable that makes
+    one (so that a passing check formats nothing)."""
     if not cond:
-        raise ValueError(msg)
+        raise ValueError(msg() if callable(msg) else msg)
 
 
 def _pool_geometry(pool):
@@ -170,24 +172,30 @@ def _pool_geometry(pool):
 
 
 def _check_tensor(name, t, dtype, ndim):
-    _need(t is not None, f"{name} is required")
-    _need(t.dtype == dtype, f"{name} must be {dtype}, got {t.dtype}")
-    _need(t.dim() == ndim, f"{name} must have {ndim} dimensions, got shape {tuple(t.shape)}")
+    """The tensor's shape, after checking that it exists, has this dtype and
+    this many dimensions."""
+    if t is None:
+        raise ValueError(f"{name} is required")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    shape = t.shape
+    if len(shape) != ndim:
+        raise ValueError(f"{name} must have {ndim} dimensions, got shape {tuple(shape)}")
+    return shape
 
 
 def _check_cache_write_args(pool, k_new, v_new, slot_mapping):
     """k_new, v_new bf16 [>= T][Hkv][d]; slot_mapping int64 [T]."""
     import torch
-    _check_tensor("slot_mapping", slot_mapping, torch.int64, 1)
-    T = slot_mapping.shape[0]
+    T = _check_tensor("slot_mapping", slot_mapping, torch.int64, 1)[0]
     geo = _pool_geometry(pool)
     for name, t in (("k_new", k_new), ("v_new", v_new)):
-        _check_tensor(name, t, torch.bfloat16, 3)
-        _need(t.shape[0] >= T, f"{name} has {t.shape[0]} rows for {T} slots")
+        ts = _check_tensor(name, t, torch.bfloat16, 3)
+        _need(ts[0] >= T, lambda: f"{name} has {ts[0]} rows for {T} slots")
         if geo is not None:
-            _need(tuple(t.shape[1:]) == geo[1:],
-                  f"{name} rows must be [num_kv_heads][head_dim] = {list(geo[1:])}, "
-                  f"got {list(t.shape[1:])}")
+            _need(ts[1] == geo[1] and ts[2] == geo[2],
+                  lambda: f"{name} rows must be [num_kv_heads][head_dim] = {list(geo[1:])}, "
+                  f"got {list(ts[1:])}")
 
 
 def _check_attn_args(pool, q, out, lse, context_lens, block_table, min_q_rows):
@@ -195,26 +203,25 @@ def _check_attn_args(pool, q, out, lse, context_lens, block_table, min_q_rows):
     multiple of its kv heads; out bf16 with q's row layout; lse fp32 [.][Hq]
     or None; context_lens int32 [R]; block_table int32 [>= R][max_blocks]."""
     import torch
-    _check_tensor("context_lens", context_lens, torch.int32, 1)
-    R = context_lens.shape[0]
-    _check_tensor("block_table", block_table, torch.int32, 2)
-    _need(block_table.shape[0] >= R, f"block_table has {block_table.shape[0]} rows for {R} requests")
-    _need(block_table.shape[1] >= 1, "block_table needs at least one column")
-    _check_tensor("q", q, torch.bfloat16, 3)
-    _need(q.shape[0] >= min_q_rows, f"q has {q.shape[0]} rows, {min_q_rows} needed")
+    R = _check_tensor("context_lens", context_lens, torch.int32, 1)[0]
+    bs = _check_tensor("block_table", block_table, torch.int32, 2)
+    _need(bs[0] >= R, lambda: f"block_table has {bs[0]} rows for {R} requests")
+    _need(bs[1] >= 1, "block_table needs at least one column")
+    qs = _check_tensor("q", q, torch.bfloat16, 3)
+    _need(qs[0] >= min_q_rows, lambda: f"q has {qs[0]} rows, {min_q_rows} needed")
     geo = _pool_geometry(pool)
     if geo is not None:
-        _need(q.shape[2] == geo[2], f"q head dim {q.shape[2]} != the pool's {geo[2]}")
-        _need(q.shape[1] % geo[1] == 0,
-              f"{q.shape[1]} query heads are not a multiple of the pool's {geo[1]} kv heads")
-    _check_tensor("out", out, torch.bfloat16, 3)
-    _need(tuple(out.shape[1:]) == tuple(q.shape[1:]),
-          f"out rows must be {list(q.shape[1:])}, got {list(out.shape[1:])}")
-    _need(out.shape[0] >= min_q_rows, f"out has {out.shape[0]} rows, {min_q_rows} needed")
+        _need(qs[2] == geo[2], lambda: f"q head dim {qs[2]} != the pool's {geo[2]}")
+        _need(qs[1] % geo[1] == 0,
+              lambda: f"{qs[1]} query heads are not a multiple of the pool's {geo[1]} kv heads")
+    os_ = _check_tensor("out", out, torch.bfloat16, 3)
+    _need(os_[1] == qs[1] and os_[2] == qs[2],
+          lambda: f"out rows must be {list(qs[1:])}, got {list(os_[1:])}")
+    _need(os_[0] >= min_q_rows, lambda: f"out has {os_[0]} rows, {min_q_rows} needed")
     if lse is not None:
-        _check_tensor("lse", lse, torch.float32, 2)
-        _need(lse.shape[1] == q.shape[1], f"lse must have {q.shape[1]} columns, got {lse.shape[1]}")
-        _need(lse.shape[0] >= min_q_rows, f"lse has {lse.shape[0]} rows, {min_q_rows} needed")
+        ls = _check_tensor("lse", lse, torch.float32, 2)
+        _need(ls[1] == qs[1], lambda: f"lse must have {qs[1]} columns, got {ls[1]}")
+        _need(ls[0] >= min_q_rows, lambda: f"lse has {ls[0]} rows, {min_q_rows} needed")
 
 
 def _stream(stream):
@@ -237,7 +244,7 @@ def kv_pool_create(num_blocks: int, num_kv_heads: int, head_dim: int, k_cache=No
         shape = (num_blocks, num_kv_heads, block_size, head_dim)
         for name, t in (("k_cache", k_cache), ("v_cache", v_cache)):
             _check_tensor(name, t, torch.bfloat16, 4)
-            _need(tuple(t.shape) == shape, f"{name} must have shape {list(shape)}, got {list(t.shape)}")
+            _need(tuple(t.shape) == shape, lambda: f"{name} must have shape {list(shape)}, got {list(t.shape)}")
     h = ctypes.c_void_p()
     _check(load().kv_pool_create(ctypes.byref(desc), _dptr(k_cache), _dptr(v_cache),
                                  ctypes.byref(h)))
@@ -317,12 +324,12 @@ def paged_attn_prefill(pool, q, out, lse, cu_seqlens_q, context_lens, block_tabl
                        max_seqlen_q: int, scale: float, stream=None):
     import torch
     _check_attn_args(pool, q, out, lse, context_lens, block_table, 0)
-    _need(tuple(out.shape) == tuple(q.shape), f"out must have q's shape {list(q.shape)}")
+    _need(tuple(out.shape) == tuple(q.shape), lambda: f"out must have q's shape {list(q.shape)}")
     if lse is not None:
-        _need(lse.shape[0] == q.shape[0], f"lse must have {q.shape[0]} rows")
+        _need(lse.shape[0] == q.shape[0], lambda: f"lse must have {q.shape[0]} rows")
     _check_tensor("cu_seqlens_q", cu_seqlens_q, torch.int32, 1)
     _need(cu_seqlens_q.shape[0] == context_lens.shape[0] + 1,
-          f"cu_seqlens_q must have {context_lens.shape[0] + 1} entries")
+          lambda: f"cu_seqlens_q must have {context_lens.shape[0] + 1} entries")
     _check(load().paged_attn_prefill(
         pool, _dptr(q), _dptr(out), _dptr(lse), _dptr(cu_seqlens_q), _dptr(context_lens),
         _dptr(block_table), int(block_table.shape[1]), int(context_lens.shape[0]),
@@ -336,7 +343,7 @@ def make_prefix_groups(num_groups=0, max_group_blocks=0, max_group_members=0, gr
                        ("group_blocks", group_blocks, num_groups), ("group_of_req", group_of_req, 0)):
         if t is not None or num_groups > 0:
             _check_tensor(name, t, torch.int32, 1)
-            _need(t.shape[0] >= n, f"{name} has {t.shape[0]} entries, {n} needed")
+            _need(t.shape[0] >= n, lambda: f"{name} has {t.shape[0]} entries, {n} needed")
     return PrefixGroups(int(num_groups), int(max_group_blocks), int(max_group_members), 0,
                         _dptr(group_start), _dptr(member_req), _dptr(group_blocks),
                         _dptr(group_of_req))
@@ -398,26 +405,26 @@ def _check_step_args(pool, host_in, dev_in, layout, block_table, num_q_heads, ou
     device tensors they receive."""
     import torch
     for name, t in (("host_in", host_in), ("dev_in", dev_in)):
-        _need(t is not None, f"{name} is required")
+        _need(t is not None, lambda: f"{name} is required")
         nbytes = t.numel() * t.element_size()
-        _need(nbytes >= layout.bytes, f"{name} holds {nbytes} bytes, the layout needs {layout.bytes}")
+        _need(nbytes >= layout.bytes, lambda: f"{name} holds {nbytes} bytes, the layout needs {layout.bytes}")
     _check_tensor("block_table", block_table, torch.int32, 2)
     R = block_table.shape[0]
     _check_tensor("out", out, torch.bfloat16, 3)
     _need(out.shape[0] >= R and out.shape[1] == num_q_heads,
-          f"out must be [>= {R}][{num_q_heads}][head_dim], got {list(out.shape)}")
+          lambda: f"out must be [>= {R}][{num_q_heads}][head_dim], got {list(out.shape)}")
     geo = _pool_geometry(pool)
     if geo is not None:
-        _need(out.shape[2] == geo[2], f"out head dim {out.shape[2]} != the pool's {geo[2]}")
+        _need(out.shape[2] == geo[2], lambda: f"out head dim {out.shape[2]} != the pool's {geo[2]}")
     if lse is not None:
         _check_tensor("lse", lse, torch.float32, 2)
         _need(lse.shape[0] >= R and lse.shape[1] == num_q_heads,
-              f"lse must be [>= {R}][{num_q_heads}], got {list(lse.shape)}")
+              lambda: f"lse must be [>= {R}][{num_q_heads}], got {list(lse.shape)}")
     for name, h, d in (("host_out", host_out, out), ("host_lse", host_lse, lse)):
         if h is not None:
-            _need(d is not None, f"{name} needs its device tensor")
+            _need(d is not None, lambda: f"{name} needs its device tensor")
             _need(h.dtype == d.dtype and tuple(h.shape) == tuple(d.shape),
-                  f"{name} must match its device tensor ({d.dtype} {list(d.shape)}), "
+                  lambda: f"{name} must match its device tensor ({d.dtype} {list(d.shape)}), "
                   f"got {h.dtype} {list(h.shape)}")
 
 
