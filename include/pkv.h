@@ -12,6 +12,8 @@
  * Contents: the block pool and its reference counts (kv_pool_*), slot
  * mapping (kv_slot_mapping), the prefix-caching index (pkv_prefix_cache_*)
  * and the prefix groups of a decode batch (pkv_prefix_groups_build),
+ * the adapter-first, length-bucketed dispatch of a multi-adapter request
+ * (pkv_lora_dispatch),
  * the cache write (kv_cache_write), suffix prefill (paged_attn_prefill),
  * decode (paged_attn_decode; without a caller workspace:
  * paged_attn_decode_noalloc; one host-driven step with its copies:
@@ -234,6 +236,30 @@ int pkv_prefix_groups_build(const int32_t *block_table, int32_t max_blocks, int3
                             int32_t *member_req_out, int32_t *group_blocks_out,
                             int32_t *num_groups_out, int32_t *max_group_blocks_out,
                             int32_t *max_group_members_out);
+
+/* ---- multi-adapter dispatch (host) ---------------------------------------- */
+
+/* Batches of a request whose items go to different LoRA adapters (Sec. 5.6:
+ * group the items by adapter, bucket each group by prompt length, run each
+ * bucket as one batch call, return the results in request order).
+ *  adapter_id, prompt_len: host int32 [n], both >= 0.
+ *  bucket_edges: host int32 [n_edges], strictly ascending (may be NULL when
+ *    n_edges is 0); an item of length L goes to bucket
+ *    #{j : L >= bucket_edges[j]} (edges {512, 2048}: short, medium, long).
+ *  max_batch: > 0 caps a batch at that many items (a larger bucket runs as
+ *    consecutive batches, the last one shorter); 0 leaves buckets whole.
+ * Order: adapters by their first item in the request, buckets of an adapter
+ * from the shortest range up, items of a bucket in request order.
+ * Outputs (host, caller-sized): order_out [n] (the request index of the k-th
+ * item executed: result k belongs to item order_out[k]), batch_start_out
+ * [n + 1] (batch b is order_out[batch_start_out[b] .. batch_start_out[b+1])),
+ * batch_adapter_out [n], batch_bucket_out [n], *n_batches_out.
+ * Errors: INVALID_ARG (negative sizes, ids or lengths; edges not ascending);
+ * nothing is written then except the message. */
+int pkv_lora_dispatch(const int32_t *adapter_id, const int32_t *prompt_len, int32_t n,
+                      const int32_t *bucket_edges, int32_t n_edges, int32_t max_batch,
+                      int32_t *order_out, int32_t *batch_start_out, int32_t *batch_adapter_out,
+                      int32_t *batch_bucket_out, int32_t *n_batches_out);
 
 /* ---- a3: cache write (device) ------------------------------------------- */
 

@@ -18,7 +18,7 @@ SRC = os.path.join(HERE, "csrc")
 OUT = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT, "libpkv.so")
 ROOT = os.path.dirname(HERE)
-SOURCES = ["pkv_api.cpp", "prefix_cache.cpp", "cache_write.cu", "decode.cu", "prefill.cu",
+SOURCES = ["pkv_api.cpp", "prefix_cache.cpp", "lora_dispatch.cpp", "cache_write.cu", "decode.cu", "prefill.cu",
            "decode_noalloc.cu", "selftest.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",

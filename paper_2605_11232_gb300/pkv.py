@@ -42,7 +42,7 @@ EXPORTS = [
     "pkv_trace_read", "pkv_check_device_errors", "pkv_last_error", "pkv_prefix_cache_create",
     "pkv_prefix_cache_destroy", "pkv_prefix_cache_match", "pkv_prefix_cache_insert",
     "pkv_prefix_cache_evict", "pkv_prefix_cache_size", "pkv_prefix_groups_build",
-    "pkv_selftest_wait_timeout",
+    "pkv_selftest_wait_timeout", "pkv_lora_dispatch",
 ]
 
 
@@ -123,6 +123,7 @@ def load(path: str | None = None):
         "pkv_prefix_cache_size": [V, P],
         "pkv_prefix_groups_build": [P, i32, i32, P, i32, P, P, P, P, P, P, P],
         "pkv_selftest_wait_timeout": [V, i32, V],
+        "pkv_lora_dispatch": [P, P, i32, P, i32, i32, P, P, P, P, P],
         "pkv_trace_read": [V, P, i32, P],
     }
     for name, args in sig.items():
@@ -542,6 +543,31 @@ def pkv_prefix_groups_build(block_table, context_lens, min_shared_blocks: int = 
     return dict(group_of_req=gor[:R], group_start=gstart[:G + 1], member_req=members[:int(gstart[G])],
                 group_blocks=gblocks[:G], num_groups=G, max_group_blocks=int(cnt[1]),
                 max_group_members=int(cnt[2]))
+
+
+# ---- multi-adapter dispatch (host) -------------------------------------------
+
+def pkv_lora_dispatch(adapter_id, prompt_len, bucket_edges=(), max_batch: int = 0):
+    """Batches of a multi-adapter request: (order, batches) with order[k] the
+    request index of the k-th item executed and batches a list of
+    (adapter_id, bucket, start, stop) over order."""
+    a = np.ascontiguousarray(adapter_id, np.int32)
+    n_ = np.ascontiguousarray(prompt_len, np.int32)
+    e = np.ascontiguousarray(bucket_edges, np.int32)
+    if a.shape != n_.shape or a.ndim != 1:
+        raise ValueError("one adapter id and one prompt length per item")
+    n = len(a)
+    order = np.zeros(max(n, 1), np.int32)
+    start = np.zeros(n + 1, np.int32)
+    adp = np.zeros(max(n, 1), np.int32)
+    bkt = np.zeros(max(n, 1), np.int32)
+    nb = np.zeros(1, np.int32)
+    _check(load().pkv_lora_dispatch(_np_ptr(a), _np_ptr(n_), n, _np_ptr(e) if len(e) else None,
+                                    len(e), int(max_batch), _np_ptr(order), _np_ptr(start),
+                                    _np_ptr(adp), _np_ptr(bkt), _np_ptr(nb)))
+    k = int(nb[0])
+    return order[:n].tolist(), [(int(adp[b]), int(bkt[b]), int(start[b]), int(start[b + 1]))
+                                for b in range(k)]
 
 
 def pkv_selftest_wait_timeout(pool, limit_us: int = 1000, stream=None):

@@ -1,7 +1,8 @@
 /* A plain C11 client of the library's host-side calls (no GPU): a pool
  * without device caches, block allocation, slot mapping, the prefix-caching
- * index and the prefix-group builder.  Prints "ok" on success; any failure
- * prints the call and its message and exits non-zero. */
+ * index, the prefix-group builder and the multi-adapter dispatch.  Prints
+ * "ok" on success; any failure prints the call and its message and exits
+ * non-zero. */
 #include <stdio.h>
 #include <stdlib.h>
 
@@ -67,6 +68,21 @@ int main(void) {
     EXPECT(nfree == 64);
     CHECK(pkv_prefix_cache_destroy(cache));
     CHECK(kv_pool_destroy(pool));
+
+    /* a 12-prompt request over four adapters (4/3/3/2), short / medium / long */
+    {
+        const int32_t adapter[12] = {22, 11, 33, 11, 44, 22, 11, 33, 22, 44, 11, 33};
+        const int32_t len[12] = {3000, 400, 800, 2500, 120, 450, 380, 700, 2048, 511, 512, 2047};
+        const int32_t edges[2] = {512, 2048};
+        const int32_t want_order[12] = {5, 0, 8, 1, 6, 10, 3, 2, 7, 11, 4, 9};
+        const int32_t want_start[8] = {0, 1, 3, 5, 6, 7, 10, 12};
+        int32_t order[12], start[13], badp[12], bbkt[12], nb = 0;
+        CHECK(pkv_lora_dispatch(adapter, len, 12, edges, 2, 0, order, start, badp, bbkt, &nb));
+        EXPECT(nb == 7);
+        for (int k = 0; k < 12; ++k) EXPECT(order[k] == want_order[k]);
+        for (int b = 0; b <= 7; ++b) EXPECT(start[b] == want_start[b]);
+        EXPECT(badp[0] == 22 && bbkt[0] == 0 && badp[1] == 22 && bbkt[1] == 2 && badp[6] == 44);
+    }
 
     /* every declared entry point resolves */
     void *entries[] = {(void *)kv_cache_write, (void *)paged_attn_prefill, (void *)paged_attn_decode,

@@ -96,3 +96,51 @@ def test_definition_invariants_and_padding(seed):
     if not max_batch:
         o0, b0 = D.dispatch(adapter, length)
         assert D.padded_tokens(length, order, batches) <= D.padded_tokens(length, o0, b0)
+
+
+# ---- the library (CPU: host code of libpkv.so) ------------------------------
+
+def _lib():
+    from _lib import built_lib
+    from paper_2605_11232_gb300 import pkv
+    built_lib()
+    return pkv
+
+
+def test_library_hand_example():
+    pkv = _lib()
+    for mb in (0, 1, 2, 3, 100):
+        assert pkv.pkv_lora_dispatch(ADAPTER, LENGTH, EDGES, mb) == D.dispatch(ADAPTER, LENGTH, EDGES, mb)
+    order, batches = pkv.pkv_lora_dispatch(ADAPTER, LENGTH, EDGES)
+    assert _as_lists(order, batches) == HAND_BATCHES
+
+
+@pytest.mark.parametrize("seed", range(30))
+def test_library_matches_definition(seed):
+    pkv = _lib()
+    rng = np.random.default_rng(100 + seed)
+    n = int(rng.integers(0, 300))
+    adapter = rng.integers(0, int(rng.integers(1, 40)), n).tolist()
+    # a mix of short classification, medium summary and long extraction prompts
+    length = np.where(rng.random(n) < 0.5, rng.integers(16, 512, n),
+                      np.where(rng.random(n) < 0.6, rng.integers(512, 2048, n),
+                               rng.integers(2048, 8192, n))).tolist()
+    edges = sorted(set(rng.integers(1, 8192, int(rng.integers(0, 6))).tolist()))
+    max_batch = int(rng.integers(0, 9))
+    got = pkv.pkv_lora_dispatch(adapter, length, edges, max_batch)
+    assert got == D.dispatch(adapter, length, edges, max_batch)
+    _check_invariants(adapter, length, edges, max_batch, *got)
+
+
+def test_library_degenerate_and_errors():
+    pkv = _lib()
+    assert pkv.pkv_lora_dispatch([], []) == ([], [])
+    assert pkv.pkv_lora_dispatch([5], [0], [1]) == ([0], [(5, 0, 0, 1)])
+    assert pkv.pkv_lora_dispatch([5, 6], [2**31 - 1, 0], [1, 2**31 - 1]) == \
+        D.dispatch([5, 6], [2**31 - 1, 0], [1, 2**31 - 1])
+    for args in (([1], [5], [10, 10]), ([1], [-5], []), ([-1], [5], []), ([1], [5], [3, 2])):
+        with pytest.raises(pkv.PkvError) as e:
+            pkv.pkv_lora_dispatch(*args)
+        assert e.value.code == pkv.PKV_ERR_INVALID_ARG
+    with pytest.raises(pkv.PkvError):
+        pkv.pkv_lora_dispatch([1, 2], [3, 4], [], -1)
