@@ -170,6 +170,18 @@ int kv_slot_mapping(pkv_pool_t pool, const int32_t *block_table, int32_t max_blo
                     const int32_t *context_lens, const int32_t *new_lens, int32_t num_requests,
                     int64_t *slots_out);
 
+/* Host check of a batch's block tables before a launch (the kernels check
+ * every block id they read as well, latching DEVICE_BOUNDS): for each request
+ * r, the entries a kernel reads, block_table[r][0 .. ceil(context_lens[r] /
+ * 16)), must name allocated blocks of the pool; later entries are never read
+ * and are not checked.  block_table: host int32 [num_requests][max_blocks];
+ * context_lens: host int32 [num_requests].  Returns PKV_OK, INVALID_ARG (a
+ * negative context or one longer than 16 * max_blocks) or REFCOUNT (an id
+ * outside the pool or a free block); *bad_request_out (may be NULL) gets the
+ * first offending request, -1 when none. */
+int pkv_check_block_table(pkv_pool_t pool, const int32_t *block_table, int32_t max_blocks,
+                          int32_t num_requests, const int32_t *context_lens, int32_t *bad_request_out);
+
 /* ---- automatic prefix caching (host) -------------------------------------- */
 
 /* An index of cached full blocks of a pool, keyed by token prefix: the prefix

@@ -353,6 +353,39 @@ int kv_slot_mapping(pkv_pool_t pool, const int32_t *block_table, int32_t max_blo
     return ok();
 }
 
+int pkv_check_block_table(pkv_pool_t pool, const int32_t *block_table, int32_t max_blocks,
+                          int32_t num_requests, const int32_t *context_lens, int32_t *bad_request_out) {
+    if (bad_request_out) *bad_request_out = -1;
+    if (!pool || num_requests < 0 || max_blocks <= 0 ||
+        (num_requests > 0 && (!block_table || !context_lens)))
+        return fail(PKV_ERR_INVALID_ARG, "bad arguments");
+    for (int32_t r = 0; r < num_requests; ++r) {
+        const int32_t L = context_lens[r];
+        const int64_t nblk = ((int64_t)L + 15) / 16;
+        int rc = PKV_OK;
+        if (L < 0 || nblk > max_blocks) {
+            rc = fail(PKV_ERR_INVALID_ARG, "request %d: context %d does not fit %d table entries", r, L,
+                      max_blocks);
+        } else {
+            const int32_t *row = block_table + (int64_t)r * max_blocks;
+            for (int64_t j = 0; j < nblk && rc == PKV_OK; ++j) {
+                const int32_t id = row[j];
+                if (id < 0 || id >= pool->desc.num_blocks)
+                    rc = fail(PKV_ERR_REFCOUNT, "request %d: entry %lld holds block id %d, outside the pool",
+                              r, (long long)j, id);
+                else if (pool->refcnt[id] == 0)
+                    rc = fail(PKV_ERR_REFCOUNT, "request %d: entry %lld holds free block %d", r,
+                              (long long)j, id);
+            }
+        }
+        if (rc != PKV_OK) {
+            if (bad_request_out) *bad_request_out = r;
+            return rc;
+        }
+    }
+    return ok();
+}
+
 int kv_cache_write(pkv_pool_t pool, const void *k_new, const void *v_new,
                    const int64_t *slot_mapping, int32_t num_tokens, pkv_stream_t stream) {
     int rc = check_kernel_pool(pool);

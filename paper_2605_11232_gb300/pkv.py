@@ -42,7 +42,7 @@ EXPORTS = [
     "pkv_trace_read", "pkv_check_device_errors", "pkv_last_error", "pkv_prefix_cache_create",
     "pkv_prefix_cache_destroy", "pkv_prefix_cache_match", "pkv_prefix_cache_insert",
     "pkv_prefix_cache_evict", "pkv_prefix_cache_size", "pkv_prefix_groups_build",
-    "pkv_selftest_wait_timeout", "pkv_lora_dispatch",
+    "pkv_selftest_wait_timeout", "pkv_lora_dispatch", "pkv_check_block_table",
 ]
 
 
@@ -124,6 +124,7 @@ def load(path: str | None = None):
         "pkv_prefix_groups_build": [P, i32, i32, P, i32, P, P, P, P, P, P, P],
         "pkv_selftest_wait_timeout": [V, i32, V],
         "pkv_lora_dispatch": [P, P, i32, P, i32, i32, P, P, P, P, P],
+        "pkv_check_block_table": [V, P, i32, i32, P, P],
         "pkv_trace_read": [V, P, i32, P],
     }
     for name, args in sig.items():
@@ -311,6 +312,22 @@ def kv_slot_mapping(pool, block_table: np.ndarray, context_lens, new_lens,
     _check(load().kv_slot_mapping(pool, _np_ptr(table), table.shape[1], _np_ptr(ctx),
                                   _np_ptr(new), len(ctx), _np_ptr(out)))
     return out[:n]
+
+
+def pkv_check_block_table(pool, block_table, context_lens) -> None:
+    """Raise PkvError (with .bad_request) unless every table entry a kernel
+    will read names an allocated block of the pool."""
+    table = np.ascontiguousarray(block_table, np.int32)
+    ctx = np.ascontiguousarray(context_lens, np.int32)
+    if table.ndim != 2 or table.shape[0] != len(ctx):
+        raise ValueError("block_table must be [num_requests][max_blocks]")
+    bad = np.zeros(1, np.int32)
+    rc = load().pkv_check_block_table(pool, _np_ptr(table), table.shape[1], len(ctx), _np_ptr(ctx),
+                                      _np_ptr(bad))
+    if rc != PKV_OK:
+        err = PkvError(rc, pkv_last_error())
+        err.bad_request = int(bad[0])
+        raise err
 
 
 # ---- a3-a7: kernels ---------------------------------------------------------

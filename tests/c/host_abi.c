@@ -57,6 +57,9 @@ int main(void) {
     CHECK(pkv_prefix_groups_build(&table[0][0], 3, 2, ctx, 1, gor, gstart, members, gblocks, &G, &mgb,
                                   &mgm));
     EXPECT(G == 1 && gblocks[0] == 2 && gor[0] == 0 && gor[1] == 0 && mgm == 2);
+    int32_t bad_req = 0;
+    CHECK(pkv_check_block_table(pool, &table[0][0], 3, 2, ctx, &bad_req));
+    EXPECT(bad_req == -1);
 
     /* requests end; the index keeps the shared blocks until they are evicted */
     CHECK(kv_pool_release(pool, row_a, 3));

@@ -153,3 +153,36 @@ def test_paged_waste_below_paper_bound(name):
     fig = json.load(open(os.path.join(GOLDEN, "paper_figures.json")))
     w = make_workload(name, values=False)
     assert _paged_waste(w) < fig["paged_kv_waste_upper_bound"]["value"]
+
+
+def test_check_block_table_on_the_host():
+    """Every entry a kernel reads (the first ceil(L / 16) of a row) must name
+    an allocated block; later entries are not read and not checked."""
+    built_lib()
+    p = pkv.kv_pool_create(32, 2, 64)
+    pre = pkv.kv_pool_alloc(p, 2)
+    rows = [pkv.kv_pool_alloc_sequence(p, pre, n) for n in (3, 4)]
+    table = np.full((2, 6), -1, np.int32)
+    for r, row in enumerate(rows):
+        table[r, : len(row)] = row
+    ctx = np.array([40, 64], np.int32)                  # 3 and 4 blocks
+    pkv.pkv_check_block_table(p, table, ctx)            # valid; -1 padding past the context
+    table[1, 5] = 999                                   # past request 1's context: not read
+    pkv.pkv_check_block_table(p, table, ctx)
+    for r, j, v, code in ((1, 3, 999, pkv.PKV_ERR_REFCOUNT), (0, 2, -1, pkv.PKV_ERR_REFCOUNT),
+                          (1, 0, 31, pkv.PKV_ERR_REFCOUNT)):     # block 31 is free
+        bad = table.copy()
+        bad[r, j] = v
+        with pytest.raises(pkv.PkvError) as e:
+            pkv.pkv_check_block_table(p, bad, ctx)
+        assert e.value.code == code and e.value.bad_request == r
+    for c, code in (([40, 97], pkv.PKV_ERR_INVALID_ARG), ([-1, 64], pkv.PKV_ERR_INVALID_ARG)):
+        with pytest.raises(pkv.PkvError) as e:
+            pkv.pkv_check_block_table(p, table, np.array(c, np.int32))
+        assert e.value.code == code
+    # a released row's private blocks are free again: the stale row is refused
+    pkv.kv_pool_release(p, rows[1])
+    with pytest.raises(pkv.PkvError) as e:
+        pkv.pkv_check_block_table(p, table, ctx)
+    assert e.value.bad_request == 1
+    pkv.kv_pool_destroy(p)
