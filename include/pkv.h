@@ -164,8 +164,8 @@ int kv_pool_alloc_sequence(pkv_pool_t pool, const int32_t *prefix_ids, int32_t n
  * row-major; slots_out has sum(new_lens) entries.  With a pool (non-NULL),
  * every target block must be allocated and unshared: a slot in a block with
  * reference count > 1 returns SHARED_BLOCK_WRITE (shared prefix blocks are
- * immutable), a free or out-of-range block REFCOUNT.  pool may be NULL (no
- * ownership checks). */
+ * immutable), a free block REFCOUNT, a block id outside the pool INVALID_ARG.
+ * pool may be NULL (no ownership checks). */
 int kv_slot_mapping(pkv_pool_t pool, const int32_t *block_table, int32_t max_blocks,
                     const int32_t *context_lens, const int32_t *new_lens, int32_t num_requests,
                     int64_t *slots_out);
@@ -176,9 +176,10 @@ int kv_slot_mapping(pkv_pool_t pool, const int32_t *block_table, int32_t max_blo
  * 16)), must name allocated blocks of the pool; later entries are never read
  * and are not checked.  block_table: host int32 [num_requests][max_blocks];
  * context_lens: host int32 [num_requests].  Returns PKV_OK, INVALID_ARG (a
- * negative context or one longer than 16 * max_blocks) or REFCOUNT (an id
- * outside the pool or a free block); *bad_request_out (may be NULL) gets the
- * first offending request, -1 when none. */
+ * negative context, one longer than 16 * max_blocks, or a block id outside
+ * the pool: the condition the kernels latch as DEVICE_BOUNDS) or REFCOUNT (a
+ * free block); *bad_request_out (may be NULL) gets the first offending
+ * request, -1 when none. */
 int pkv_check_block_table(pkv_pool_t pool, const int32_t *block_table, int32_t max_blocks,
                           int32_t num_requests, const int32_t *context_lens, int32_t *bad_request_out);
 
@@ -337,6 +338,25 @@ int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
                       int32_t max_blocks, int32_t num_requests, int32_t num_q_heads,
                       float scale, const pkv_prefix_groups *groups, void *workspace,
                       size_t workspace_bytes, pkv_stream_t stream);
+
+/* paged_attn_decode with the cache write of the query tokens fused in: each
+ * request's own key and value (the token it decodes, at position
+ * context_lens[r] - 1) are stored into the pool by the decode kernels instead
+ * of a kv_cache_write launch beforehand, then all context_lens[r] keys are
+ * attended to as by paged_attn_decode (Sec. 5.3's decode step; Sec. 5.4's
+ * paged cache).  The result, and the pool afterwards, equal kv_cache_write of
+ * those tokens to slots block_table[r][(L - 1) / 16] * 16 + (L - 1) % 16
+ * followed by paged_attn_decode.
+ *  k_new, v_new: device bf16 [R][num_kv_heads][head_dim], 16-byte aligned.
+ *  The block holding position L - 1 must be the request's own (reference
+ *  count 1; the decode requires its last block private in any case).
+ * Every other argument, the workspace and the errors are those of
+ * paged_attn_decode. */
+int paged_attn_decode_append(pkv_pool_t pool, const void *q, const void *k_new, const void *v_new,
+                             void *out, float *lse, const int32_t *context_lens,
+                             const int32_t *block_table, int32_t max_blocks, int32_t num_requests,
+                             int32_t num_q_heads, float scale, const pkv_prefix_groups *groups,
+                             void *workspace, size_t workspace_bytes, pkv_stream_t stream);
 
 /* ---- a decode step from host memory --------------------------------------- */
 

@@ -228,6 +228,16 @@ def run_decode(b: Batch, out: torch.Tensor, lse, ws: torch.Tensor, use_groups: b
                           b.w.scale, b.groups if use_groups else None, ws, stream)
 
 
+def run_decode_append(b: Batch, out: torch.Tensor, lse, ws: torch.Tensor, use_groups: bool = True,
+                      stream=None):
+    """The decode subset's cache write and attention in one call: each decode
+    request's new K/V row is stored by the decode kernels."""
+    rows = new_token_rows(b.w, b.dec)
+    pkv.paged_attn_decode_append(b.pool, b.q[rows], b.k_new[rows], b.v_new[rows], out, lse,
+                                 b.context_lens[b.dec], b.table[b.dec], b.w.scale,
+                                 b.groups if use_groups else None, ws, stream)
+
+
 def run_prefill(b: Batch, out: torch.Tensor, lse, stream=None):
     rows = new_token_rows(b.w, b.pre)
     pkv.paged_attn_prefill(b.pool, b.q[rows], out, lse, b.cu_pre, b.context_lens[b.pre],

@@ -8,106 +8,127 @@
 //
 // Work split ("pieces").  The private blocks of all (request, kv head) pairs
 // form one stream of W blocks, segment (r, h) after segment.  Warp w of the
-// persistent grid takes blocks [w*per, (w+1)*per) of that stream, so every
-// warp moves the same number of bytes whatever the length mix; a warp that
-// crosses a segment boundary emits one unnormalised partial (O, m, l) per
-// segment it touches.  The combine kernel merges a head's partials with
-// log-sum-exp weights.
+// grid takes the contiguous range [w*per, (w+1)*per) of that stream, so every
+// warp moves the same number of bytes whatever the length mix; a warp whose
+// range crosses segment boundaries emits one unnormalised partial (O, m, l)
+// per segment it touches.  The combine kernel merges a head's partials with
+// log-sum-exp weights.  The grid covers the SMs the shared-prefix pass leaves
+// free (all of them without one), so all warps start together and end
+// together.
 //
-// Inner loop (one 16-token block per step, per warp):
+// Data path (per warp).  The (block, kv head) K and V tiles of the warp's
+// range are copied by TMA, with the 128-byte swizzle, into a ring of stages
+// in shared memory, issued by the warp itself a few blocks ahead of the one
+// it computes on; the ring runs on across piece boundaries, and the piece
+// metadata (request, head, shared-block offset, block ids) is looked up ahead
+// of the copies, so a new segment costs no pipeline restart.
+//
+// Inner loop (one 16-token block per step):
 //   S^T[16 keys x 8 heads] = K_blk[16 x d] . Q^T[d x 8]   (mma m16n8k16, A = K)
 //   online softmax per head column (shuffles across the 8 row groups)
 //   O^T[d x 8] += V_blk^T[d x 16] . P^T[16 x 8]           (A = V^T, B = P^T)
-// K and V are read with 16-byte loads straight into registers in the order
-// the mma fragments need: the head dimension is a contraction index for
-// Q.K and the key index one for P.V, so both may be permuted freely as long
-// as both operands use the same permutation.  The S^T accumulator becomes the
-// P^T operand through one movmatrix transpose per 8x8 quadrant; the key order
-// sigma() of the QK^T rows is chosen so that the transposed fragments land on
-// exactly the keys each thread loaded for P.V.
+// A fragments come from the swizzled stages by ldmatrix (V through its
+// transposing form); the S^T accumulator becomes the P^T operand through one
+// movmatrix transpose per 8x8 quadrant.
+//
+// Fused write.  With the query tokens' own K/V given (paged_attn_decode_append),
+// the warp that reaches a request's last block stores the new row (position
+// L - 1) into the pool and over the stale row of its shared-memory stage
+// before computing on it, so no separate cache-write kernel precedes the pass.
 #include <math.h>
 
 #include <algorithm>
 
 #include "pkv_device.cuh"
 #include "pkv_internal.h"
+#include "tc_ptx.cuh"
 
 namespace pkv {
 
 namespace {
 
+using namespace tc;
+
 constexpr int kWarps = 8;
 constexpr int kThreads = kWarps * 32;
-constexpr int kChunksPerWarp = 2;   // work chunks per warp of the grid (balance vs. pipeline restarts)
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+constexpr uint64_t kDrainLimitNs = 200000000ull;
 
-__device__ __forceinline__ uint32_t reg_of(const uint4 &v, int i) {
-    return i == 0 ? v.x : (i == 1 ? v.y : (i == 2 ? v.z : v.w));
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2,
+                                        uint32_t &r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2,
+                                          uint32_t &r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
 }
 
-// Physical key (row of the 16-token block) behind logical QK^T row r (0..7);
-// row r + 8 is sigma(r) + 2.
-__device__ __forceinline__ int sigma(int r) { return 2 * r - (r & 1); }
+// Byte offset of 16-byte chunk c (head-dim elements 8c..8c+7) of key row
+// `row` inside a (block, head) tile as TMA lays it out: 64-column boxes of
+// 16 rows x 128 bytes, chunk position XORed with row % 8 (128-byte swizzle).
+__device__ __forceinline__ uint32_t tile_off(int row, int c) {
+    return (uint32_t)((c >> 3) * 2048 + row * 128 + (((c & 7) ^ (row & 7)) << 4));
+}
 
-template <int D>
-struct BlockRegs {
-    uint4 ka[D / 32];   // K[sigma(r)    ][chunk 4j+q]
-    uint4 kb[D / 32];   // K[sigma(r) + 2][chunk 4j+q]
-    uint4 va[4];        // V[4q+s][chunk r]       (d 8r..8r+7)
-    uint4 vb[D == 128 ? 4 : 1];   // V[4q+s][chunk 8+r] (d 64+8r..), d = 128 only
+// What the producer records for each stage when it issues the copies.
+struct SlotDesc {
+    int32_t r, h;
+    int32_t phys;      // physical block id
+    int32_t info;      // valid keys | kFirst | kLast | kWrite | kSegFirst
+    int32_t part;      // part slot of the piece's partial
+    int32_t nparts;    // part-count word of the segment (private | prefix << 16)
+    int32_t pad0, pad1;
 };
+constexpr int32_t kValidMask = 31;
+constexpr int32_t kFirst = 1 << 8;      // first block of a piece: reset the state, new Q
+constexpr int32_t kLast = 1 << 9;       // last block of a piece: emit the partial
+constexpr int32_t kWrite = 1 << 10;     // holds the request's query token: store k_new / v_new
+constexpr int32_t kSegFirst = 1 << 11;  // the piece starts the segment: write its part counts
+constexpr int32_t kWriteSoon = 1 << 12; // first block of a piece that ends with kWrite
 
-template <int D>
-__device__ __forceinline__ void load_block(BlockRegs<D> &b, const uint16_t *kt,
-                                           const uint16_t *vt, int lr, int lq) {
-    const int s0 = sigma(lr);
-#pragma unroll
-    for (int j = 0; j < D / 32; ++j) {
-        b.ka[j] = ldg_stream(kt + s0 * D + (4 * j + lq) * 8);
-        b.kb[j] = ldg_stream(kt + (s0 + 2) * D + (4 * j + lq) * 8);
-    }
-#pragma unroll
-    for (int s = 0; s < 4; ++s) {
-        b.va[s] = ldg_stream(vt + (4 * lq + s) * D + lr * 8);
-        if constexpr (D == 128) b.vb[s] = ldg_stream(vt + (4 * lq + s) * D + (8 + lr) * 8);
-    }
-}
-
-// Running state of one warp over one piece.  Thread (lr = lane/4, lq = lane%4)
-// holds heads 2lq, 2lq+1: m, l (thread-partial sum) and O^T fragments.
 template <int D>
 struct SoftmaxState {
-    float m[2];
-    float l[2];
+    float m[2];   // running max (base 2, scaled) of heads 2*(lane%4) + {0, 1}
+    float l[2];   // thread-partial sums
     float o[D / 16][4];
 };
 
+// One 16-key block from a stage: K tile at kb, V tile at vb (shared addresses).
 template <int D>
-__device__ __forceinline__ void attend_block(SoftmaxState<D> &st, BlockRegs<D> &b,
-                                             const uint32_t (&qf)[D / 32][4], int lr, int lq,
-                                             int valid_keys, float scale_log2) {
-    // S^T = K . Q^T
+__device__ __forceinline__ void attend_block(SoftmaxState<D> &st, uint32_t kb, uint32_t vb,
+                                             const uint32_t (&qf)[D / 16][2], int lane, int valid,
+                                             float scale_log2) {
     float sacc[4] = {0.f, 0.f, 0.f, 0.f};
+    {
+        // matrices (keys 0-7 | 8-15) x (head-dim chunk 2kk | 2kk+1): A fragment of K
+        const int row = (lane & 7) + ((lane >> 3) & 1) * 8;
+        const int hi = lane >> 4;
 #pragma unroll
-    for (int s = 0; s < D / 16; ++s) {
-        const int j = s >> 1, e = s & 1;
-        mma_bf16_16816(sacc, reg_of(b.ka[j], 2 * e), reg_of(b.kb[j], 2 * e),
-                       reg_of(b.ka[j], 2 * e + 1), reg_of(b.kb[j], 2 * e + 1), qf[j][2 * e],
-                       qf[j][2 * e + 1]);
+        for (int kk = 0; kk < D / 16; ++kk) {
+            uint32_t a0, a1, a2, a3;
+            ldsm_x4(kb + tile_off(row, 2 * kk + hi), a0, a1, a2, a3);
+            mma_bf16_16816(sacc, a0, a1, a2, a3, qf[kk][0], qf[kk][1]);
+        }
     }
-    const int key0 = sigma(lr), key1 = key0 + 2;
-    const bool ok0 = key0 < valid_keys, ok1 = key1 < valid_keys;
-    float s00 = ok0 ? sacc[0] * scale_log2 : -INFINITY;   // key0, head 2lq
-    float s01 = ok0 ? sacc[1] * scale_log2 : -INFINITY;   // key0, head 2lq+1
-    float s10 = ok1 ? sacc[2] * scale_log2 : -INFINITY;   // key1, head 2lq
-    float s11 = ok1 ? sacc[3] * scale_log2 : -INFINITY;   // key1, head 2lq+1
+    // thread (lane): keys lane/4 and lane/4 + 8, heads 2*(lane%4) + {0, 1}
+    const int key0 = lane >> 2, key1 = key0 + 8;
+    const bool ok0 = key0 < valid, ok1 = key1 < valid;
+    const float s00 = ok0 ? sacc[0] * scale_log2 : -INFINITY;
+    const float s01 = ok0 ? sacc[1] * scale_log2 : -INFINITY;
+    const float s10 = ok1 ? sacc[2] * scale_log2 : -INFINITY;
+    const float s11 = ok1 ? sacc[3] * scale_log2 : -INFINITY;
     float mx0 = fmaxf(s00, s10), mx1 = fmaxf(s01, s11);
 #pragma unroll
     for (int off = 4; off < 32; off <<= 1) {
         mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
         mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, off));
     }
+    // mn is finite: every processed block has at least one valid key
     const float mn0 = fmaxf(st.m[0], mx0), mn1 = fmaxf(st.m[1], mx1);
-    // mn is finite: every processed block has at least one valid key.
     const float a0 = fast_exp2(st.m[0] - mn0), a1 = fast_exp2(st.m[1] - mn1);
     st.m[0] = mn0;
     st.m[1] = mn1;
@@ -122,27 +143,35 @@ __device__ __forceinline__ void attend_block(SoftmaxState<D> &st, BlockRegs<D> &
         st.o[i][1] *= a1;
         st.o[i][3] *= a1;
     }
-    // P^T fragments: transpose the two 8x8 quadrants of P^T(key, head).
+    // P^T fragments: transpose the two 8x8 quadrants (keys 0-7, 8-15) of P
     const uint32_t t0 = movmatrix_trans(pack_bf16x2(p00, p01));
     const uint32_t t1 = movmatrix_trans(pack_bf16x2(p10, p11));
-    // Masked keys carry p = 0, but 0 * NaN would poison O: zero their V rows.
+    {
+        // matrices (head-dim chunk 2mt | 2mt+1) x (keys 0-7 | 8-15) of V^T,
+        // read from V's key rows by the transposing ldmatrix
+        const int j = lane >> 3, r = lane & 7;
+        const int key = 8 * (j >> 1) + r;
 #pragma unroll
-    for (int s = 0; s < 4; ++s) {
-        if (4 * lq + s >= valid_keys) {
-            b.va[s] = make_uint4(0, 0, 0, 0);
-            if constexpr (D == 128) b.vb[s] = make_uint4(0, 0, 0, 0);
+        for (int mt = 0; mt < D / 16; ++mt) {
+            uint32_t v0, v1, v2, v3;
+            ldsm_x4_t(vb + tile_off(key, 2 * mt + (j & 1)), v0, v1, v2, v3);
+            mma_bf16_16816(st.o[mt], v0, v1, v2, v3, t0, t1);
         }
     }
-    // O^T += V^T . P^T, one 16-row tile of the head dim per mma.
+}
+
+// Q fragments (B operand of S^T = K.Q^T) from a stage's copy of the g q-head
+// rows of (request, kv head): thread (lane) gets head lane/4, head-dim
+// elements 16kk + 2(lane%4) + {0, 1} and + 8.  Rows g..7 of the area hold
+// stale data: those heads' columns of S^T, P^T and O^T are never written out
+// (an MMA column depends on its own B column only).
+template <int D>
+__device__ __forceinline__ void load_q_smem(uint32_t (&qf)[D / 16][2], uint32_t qa, int lane) {
+    // matrices: head rows 0-7 x head-dim chunks c0 .. c0+3 (two k-steps)
+    const uint32_t row = qa + (uint32_t)(lane & 7) * (D * 2);
 #pragma unroll
-    for (int i = 0; i < D / 16; ++i) {
-        const uint4 *src = (i < 4) ? b.va : b.vb;
-        const int w = i & 3;
-        const uint32_t x0 = reg_of(src[0], w), x1 = reg_of(src[1], w);
-        const uint32_t x2 = reg_of(src[2], w), x3 = reg_of(src[3], w);
-        mma_bf16_16816(st.o[i], __byte_perm(x0, x1, 0x5410), __byte_perm(x0, x1, 0x7632),
-                       __byte_perm(x2, x3, 0x5410), __byte_perm(x2, x3, 0x7632), t0, t1);
-    }
+    for (int kk = 0; kk < D / 16; kk += 2)
+        ldsm_x4(row + (uint32_t)(2 * kk + (lane >> 3)) * 16, qf[kk][0], qf[kk][1], qf[kk + 1][0], qf[kk + 1][1]);
 }
 
 // Block-wide plan: P[r] = sum of the private block counts of requests < r,
@@ -209,165 +238,304 @@ __device__ void build_plan(int32_t *P, int32_t R, const int32_t *__restrict__ co
     __syncthreads();
 }
 
+// The split pass: per warp, a contiguous range of the block stream through a
+// TMA ring (see the file comment).
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1) decode_split_kernel(DecodeArgs a, DecodeLayout lay,
-                                                                  int32_t num_blocks_pool,
-                                                                  int32_t after_prefix) {
-    extern __shared__ int32_t P[];   // [R + 1]
+__global__ void __launch_bounds__(kThreads, 1)
+    decode_split_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
+                        const DecodeArgs a, const DecodeLayout lay, int32_t num_blocks_pool,
+                        int32_t after_prefix) {
+    constexpr int kHalves = D / 64;
+    constexpr uint32_t kTileBytes = kHalves * 2048;   // one K or V tile of a (block, kv head)
+    constexpr uint32_t kSlotBytes = 2 * kTileBytes;
+    constexpr int CPR = D / 8;                        // 16-byte chunks per key row
+    constexpr uint32_t kQBytes = 8 * D * 2;           // Q area of a stage: 8 head rows
+    const int S = lay.stages;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                ~uintptr_t(1023));
+    // K/V stages [kWarps][S] | Q areas [kWarps][S] | descriptors [kWarps][S] |
+    // full barriers [kWarps][S] | plan [R + 1]
+    const uint32_t qbase = smem_u32(smem) + (uint32_t)(kWarps * S) * kSlotBytes;
+    SlotDesc *descs = reinterpret_cast<SlotDesc *>(smem + (size_t)kWarps * S * (kSlotBytes + kQBytes));
+    uint64_t *bars = reinterpret_cast<uint64_t *>(descs + kWarps * S);
+    int32_t *P = reinterpret_cast<int32_t *>(bars + kWarps * S);
     __shared__ int32_t s_max_n;
+    __shared__ int abort_flag;
+
     // After a shared-prefix pass, which starts this kernel once it has seen
-    // the cache write complete, nothing read here is written by that pass:
-    // wait for it only before exiting (the combine needs both).  Without one,
-    // wait for the cache write first.
+    // everything before it complete, nothing read here is written by that
+    // pass: wait for it only before exiting (the combine needs both).
+    // Without one, wait for the preceding kernel first.
     if (!after_prefix) pdl_wait();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) abort_flag = 0;
+    const uint32_t mybar = smem_u32(bars + warp * S);
+    if (lane == 0) {
+        for (int s = 0; s < S; ++s) mbar_init(mybar + 8 * s, 1);
+        fence_barrier_init();
+    }
     const int32_t R = lay.R, Hkv = lay.Hkv, Hq = lay.Hq, g = lay.g;
     build_plan(P, R, a.context_lens, a.group_of_req, a.group_blocks, a.num_groups, a.max_blocks,
-               &s_max_n, a.err);
+               &s_max_n, a.err);   // ends with __syncthreads: the barriers are initialised
     const int64_t W = (int64_t)Hkv * P[R];
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
-    int64_t per = (W + nwarps * kChunksPerWarp - 1) / (nwarps * kChunksPerWarp);
+    int64_t per = (W + nwarps - 1) / nwarps;
     const int64_t need = (s_max_n - 1 + kMaxPrivateParts - 3) / (kMaxPrivateParts - 2);
     if (per < need) per = need;
     if (per < kMinBlocksPerPiece) per = kMinBlocksPerPiece;
+    const int64_t gw = (int64_t)blockIdx.x * kWarps + warp;
+    const int64_t x0 = gw * per, x1 = min(x0 + per, W);
+    const int64_t nu = x1 - x0;   // units (blocks of one kv head) of this warp
 
-    const int lane = threadIdx.x & 31;
-    const int lr = lane >> 2, lq = lane & 3;
-    const int64_t nchunks = (W + per - 1) / per;
+    if (nu > 0) {
+        float *o_part = reinterpret_cast<float *>(static_cast<char *>(a.ws) + lay.off_o);
+        float2 *ml_part = reinterpret_cast<float2 *>(static_cast<char *>(a.ws) + lay.off_ml);
+        int32_t *nparts = reinterpret_cast<int32_t *>(static_cast<char *>(a.ws) + lay.off_nparts);
+        const uint32_t ring = smem_u32(smem) + (uint32_t)(warp * S) * kSlotBytes;
+        const uint32_t qarea = qbase + (uint32_t)(warp * S) * kQBytes;
+        const uint32_t qbytes = (uint32_t)g * D * 2;
+        SlotDesc *mydesc = descs + warp * S;
+        const bool fused = a.k_new != nullptr;
 
-    const uint16_t *q = static_cast<const uint16_t *>(a.q);
-    const uint16_t *kc = static_cast<const uint16_t *>(a.k_cache);
-    const uint16_t *vc = static_cast<const uint16_t *>(a.v_cache);
-    float *o_part = reinterpret_cast<float *>(static_cast<char *>(a.ws) + lay.off_o);
-    float2 *ml_part = reinterpret_cast<float2 *>(static_cast<char *>(a.ws) + lay.off_ml);
-    int32_t *nparts = reinterpret_cast<int32_t *>(static_cast<char *>(a.ws) + lay.off_nparts);
-
-    // Chunks of `per` stream blocks are handed out by a counter, so that CTAs
-    // which start late (on SMs the prefix pass still holds) take less work.
-    for (;;) {
-      int chunk = 0;
-      if (lane == 0) chunk = atomicAdd(a.sched, 1);
-      chunk = __shfl_sync(0xffffffffu, chunk, 0);
-      if (chunk >= nchunks) break;
-      int64_t x = (int64_t)chunk * per;
-      const int64_t x_end = min(x + per, W);
-      while (x < x_end) {
-        // segment containing x: request r (largest r with P[r] <= x / Hkv), head h
-        const int64_t xr = x / Hkv;
-        int lo = 0, hi = R - 1;
-        while (lo < hi) {
-            const int mid = (lo + hi + 1) >> 1;
-            if (P[mid] <= xr) lo = mid; else hi = mid - 1;
-        }
-        const int r = lo;
-        const int32_t n = P[r + 1] - P[r];
-        const int64_t seg_base = (int64_t)Hkv * P[r];
-        const int h = (int)((x - seg_base) / n);
-        const int64_t seg_off = seg_base + (int64_t)h * n;
-        const int64_t piece_end = min(x_end, seg_off + n);
-        const int b_lo = (int)(x - seg_off), b_hi = (int)(piece_end - seg_off);
-        const int part = (int)(x / per - seg_off / per);
-
-        const int32_t L = __ldg(a.context_lens + r);
-        // shared leading blocks: the plan's private count n ends at the last block
-        const int32_t nblk = min((L + 15) >> 4, a.max_blocks);
-        const int32_t sh = max(nblk - n, 0);
-        const int32_t *trow = a.block_table + (int64_t)r * a.max_blocks;
-
-        // Q fragments of the g heads of kv head h (head lr of the group)
-        uint32_t qf[D / 32][4];
+        // ---- the warp's pieces, 32 at a time: lane k describes the piece of
+        // segment seg_base + k (segment (r, h) = r * Hkv + h)
+        int64_t seg_base;
         {
-            const bool hv = lr < g;
-            const uint16_t *qrow = q + ((int64_t)r * Hq + h * g + (hv ? lr : 0)) * D;
-#pragma unroll
-            for (int j = 0; j < D / 32; ++j) {
-                uint4 v = hv ? ldg16(qrow + (4 * j + lq) * 8) : make_uint4(0, 0, 0, 0);
-                qf[j][0] = v.x; qf[j][1] = v.y; qf[j][2] = v.z; qf[j][3] = v.w;
+            const int64_t xr = x0 / Hkv;
+            int lo = 0, hi = R - 1;
+            while (lo < hi) {
+                const int mid = (lo + hi + 1) >> 1;
+                if (P[mid] <= xr) lo = mid; else hi = mid - 1;
             }
+            const int32_t n0 = P[lo + 1] - P[lo];
+            seg_base = (int64_t)lo * Hkv + (x0 - (int64_t)Hkv * P[lo]) / n0;
+        }
+        int32_t pr = 0, ph = 0, plo = 0, phi = 0, psh = 0, pL = 0, pn = 0, ppart = 0, pnw = 0;
+        auto fill_list = [&]() {
+            const int64_t sg = seg_base + lane;
+            pr = (int32_t)(sg / Hkv);
+            ph = (int32_t)(sg - (int64_t)pr * Hkv);
+            plo = phi = 0;
+            if (pr < R) {
+                pn = P[pr + 1] - P[pr];
+                const int64_t seg_off = (int64_t)Hkv * P[pr] + (int64_t)ph * pn;
+                const int64_t lo = max(x0, seg_off), hi = min(x1, seg_off + pn);
+                if (lo < hi) {
+                    plo = (int32_t)(lo - seg_off);
+                    phi = (int32_t)(hi - seg_off);
+                    pL = __ldg(a.context_lens + pr);
+                    const int32_t nblk = min((pL + 15) >> 4, a.max_blocks);
+                    psh = max(nblk - pn, 0);
+                    ppart = lay.prefix_parts + (int32_t)(gw - seg_off / per);
+                    const int32_t n_priv = (int32_t)((seg_off + pn - 1) / per - seg_off / per + 1);
+                    const int32_t n_pre = lay.prefix_parts > 0 && a.num_groups > 0
+                                              ? min((psh + lay.prefix_blocks_per_part - 1) / lay.prefix_blocks_per_part,
+                                                    lay.prefix_parts)
+                                              : 0;
+                    pnw = n_priv | (n_pre << 16);
+                }
+            }
+        };
+        fill_list();
+
+        // block ids of a piece, 32 at a time: lane j holds block base + j
+        auto load_ids = [&](int r_, int sh_, int base, int hi) -> int32_t {
+            int32_t id = 0;
+            if (base + lane < hi) {
+                id = __ldg(a.block_table + (int64_t)r_ * a.max_blocks + sh_ + base + lane);
+                if (id < 0 || id >= num_blocks_pool) {
+                    latch_error(a.err, kDevBounds);
+                    id = 0;
+                }
+            }
+            return id;
+        };
+
+        // ---- producer cursor (warp-uniform): piece k of the list, next block b
+        int k = -1, b = 0, b_lo = 0, b_hi = 0, cr = 0, ch = 0, csh = 0, cL = 0, cn = 0, cpart = 0, cnw = 0;
+        int win_base = 0, nwin_for = -1;
+        int32_t win = 0, nwin = 0;
+        auto enter_next = [&]() {
+            ++k;
+            if (k == 32) {
+                seg_base += 32;
+                fill_list();
+                k = 0;
+                nwin_for = -1;
+            }
+            cr = __shfl_sync(0xffffffffu, pr, k);
+            ch = __shfl_sync(0xffffffffu, ph, k);
+            b_lo = __shfl_sync(0xffffffffu, plo, k);
+            b_hi = __shfl_sync(0xffffffffu, phi, k);
+            csh = __shfl_sync(0xffffffffu, psh, k);
+            cL = __shfl_sync(0xffffffffu, pL, k);
+            cn = __shfl_sync(0xffffffffu, pn, k);
+            cpart = __shfl_sync(0xffffffffu, ppart, k);
+            cnw = __shfl_sync(0xffffffffu, pnw, k);
+            b = b_lo;
+            win_base = b_lo;
+            win = nwin_for == k ? nwin : load_ids(cr, csh, b_lo, b_hi);
+            // the next piece's first ids, in flight while this piece issues
+            nwin_for = -1;
+            if (k + 1 < 32) {
+                const int r1 = __shfl_sync(0xffffffffu, pr, k + 1), sh1 = __shfl_sync(0xffffffffu, psh, k + 1);
+                const int lo1 = __shfl_sync(0xffffffffu, plo, k + 1), hi1 = __shfl_sync(0xffffffffu, phi, k + 1);
+                if (lo1 < hi1) {
+                    nwin = load_ids(r1, sh1, lo1, hi1);
+                    nwin_for = k + 1;
+                }
+            }
+        };
+        // issue the copies of the next block into stage s
+        auto produce = [&](int s) {
+            if (b == b_hi) enter_next();
+            if (b - win_base >= 32) {
+                win_base = b;
+                win = load_ids(cr, csh, b, b_hi);
+            }
+            const int32_t phys = __shfl_sync(0xffffffffu, win, b - win_base);
+            const int valid = min(16, cL - (csh + b) * 16);
+            int32_t info = valid;
+            const bool first = b == b_lo;
+            const bool write_at_end = fused && b_hi == cn && cL - (csh + cn - 1) * 16 >= 1;
+            if (first) info |= kFirst | (b_lo == 0 ? kSegFirst : 0) | (write_at_end ? kWriteSoon : 0);
+            if (b == b_hi - 1) info |= kLast;
+            if (write_at_end && b == cn - 1) info |= kWrite;
+            if (lane == 0) {
+                SlotDesc dsc;
+                dsc.r = cr; dsc.h = ch; dsc.phys = phys; dsc.info = info;
+                dsc.part = cpart; dsc.nparts = cnw; dsc.pad0 = dsc.pad1 = 0;
+                mydesc[s] = dsc;
+                const uint32_t dst = ring + (uint32_t)s * kSlotBytes, bar = mybar + 8 * s;
+                fence_proxy_async_smem();   // this stage's earlier generic reads / writes
+                mbar_arrive_expect_tx(bar, kSlotBytes + (first ? qbytes : 0u));
+                if (first)   // the piece's g q-head rows, contiguous in q
+                    bulk_load(qarea + (uint32_t)s * kQBytes,
+                              static_cast<const uint16_t *>(a.q) + ((int64_t)cr * Hq + (int64_t)ch * g) * D, qbytes, bar);
+#pragma unroll
+                for (int hf = 0; hf < kHalves; ++hf) {
+                    tma_load_4d(dst + hf * 2048, &tmk, hf * 64, 0, ch, phys, bar);
+                    tma_load_4d(dst + kTileBytes + hf * 2048, &tmv, hf * 64, 0, ch, phys, bar);
+                }
+            }
+            __syncwarp();
+            ++b;
+        };
+
+        if (lane == 0) {
+            prefetch_tmap(&tmk);
+            prefetch_tmap(&tmv);
+        }
+        const int64_t n_first = nu < S ? nu : (int64_t)S;
+        for (int s = 0; s < n_first; ++s) produce(s);
+
+        uint32_t qf[D / 16][2];
+        uint4 kvn = make_uint4(0, 0, 0, 0);   // lane < CPR: k_new chunk; < 2 CPR: v_new chunk
+        auto load_new = [&](const SlotDesc &d) {
+            if (lane < 2 * CPR) {
+                const uint16_t *src = static_cast<const uint16_t *>(lane < CPR ? a.k_new : a.v_new);
+                const int c = lane < CPR ? lane : lane - CPR;
+                kvn = ldg16(src + ((int64_t)d.r * Hkv + d.h) * D + c * 8);
+            }
+        };
+        {
+            const SlotDesc d0 = mydesc[0];
+            if (d0.info & kWriteSoon) load_new(d0);
         }
         SoftmaxState<D> st;
-        st.m[0] = st.m[1] = -INFINITY;
-        st.l[0] = st.l[1] = 0.f;
+        int s = 0;
+        uint32_t phase = 0;
+        int64_t u = 0;
+        for (; u < nu; ++u) {
+            if (!__all_sync(0xffffffffu, mbar_wait(mybar + 8 * s, phase, &abort_flag, kWaitLimitNs))) break;
+            const SlotDesc d = mydesc[s];
+            const int valid = d.info & kValidMask;
+            const uint32_t kb = ring + (uint32_t)s * kSlotBytes, vb = kb + kTileBytes;
+            if (d.info & kFirst) {
+                load_q_smem<D>(qf, qarea + (uint32_t)s * kQBytes, lane);
+                st.m[0] = st.m[1] = -INFINITY;
+                st.l[0] = st.l[1] = 0.f;
 #pragma unroll
-        for (int i = 0; i < D / 16; ++i) st.o[i][0] = st.o[i][1] = st.o[i][2] = st.o[i][3] = 0.f;
-
-        // block ids of this piece, 32 at a time, one per lane
-        int win_base = b_lo;
-        int32_t my_phys = 0;
-        auto refresh = [&](int base) {
-            win_base = base;
-            const int bi = sh + base + lane;
-            int32_t p = (base + lane < b_hi) ? __ldg(trow + bi) : 0;
-            if (p < 0 || p >= num_blocks_pool) {
-                if (base + lane < b_hi) latch_error(a.err, kDevBounds);
-                p = 0;
+                for (int i = 0; i < D / 16; ++i) st.o[i][0] = st.o[i][1] = st.o[i][2] = st.o[i][3] = 0.f;
+                if ((d.info & kSegFirst) && lane == 0) nparts[(int64_t)d.r * Hkv + d.h] = d.nparts;
             }
-            my_phys = p;
-        };
-        refresh(b_lo);
-        auto tile_of = [&](int b, const uint16_t *base) {
-            if (b - win_base >= 32) refresh(b);
-            const int32_t phys = __shfl_sync(0xffffffffu, my_phys, b - win_base);
-            return base + ((int64_t)phys * Hkv + h) * 16 * D;
-        };
-        auto valid_of = [&](int b) {
-            const int pos0 = (sh + b) * 16;
-            return min(16, L - pos0);
-        };
-
-        BlockRegs<D> b0, b1;
-        load_block<D>(b0, tile_of(b_lo, kc), tile_of(b_lo, vc), lr, lq);
-        for (int b = b_lo; b < b_hi; b += 2) {
-            if (b + 1 < b_hi) load_block<D>(b1, tile_of(b + 1, kc), tile_of(b + 1, vc), lr, lq);
-            attend_block<D>(st, b0, qf, lr, lq, valid_of(b), a.scale_log2);
-            if (b + 1 >= b_hi) break;
-            if (b + 2 < b_hi) load_block<D>(b0, tile_of(b + 2, kc), tile_of(b + 2, vc), lr, lq);
-            attend_block<D>(st, b1, qf, lr, lq, valid_of(b + 1), a.scale_log2);
-        }
-
-        // row-group reduction of the thread-partial sums
-#pragma unroll
-        for (int off = 4; off < 32; off <<= 1) {
-            st.l[0] += __shfl_xor_sync(0xffffffffu, st.l[0], off);
-            st.l[1] += __shfl_xor_sync(0xffffffffu, st.l[1], off);
-        }
-        const int slot_part = lay.prefix_parts + part;
-#pragma unroll
-        for (int c = 0; c < 2; ++c) {
-            const int hd = 2 * lq + c;
-            if (hd < g) {
-                const int64_t slot = ((int64_t)r * Hq + h * g + hd) * lay.parts_per_head + slot_part;
-                float *dst = o_part + slot * D;
-#pragma unroll
-                for (int half = 0; half < D / 64; ++half) {
-                    const int i0 = half * 4;
-                    float4 v0 = make_float4(st.o[i0][c], st.o[i0][2 + c], st.o[i0 + 1][c],
-                                            st.o[i0 + 1][2 + c]);
-                    float4 v1 = make_float4(st.o[i0 + 2][c], st.o[i0 + 2][2 + c],
-                                            st.o[i0 + 3][c], st.o[i0 + 3][2 + c]);
-                    float4 *p4 = reinterpret_cast<float4 *>(dst + half * 64 + lr * 8);
-                    p4[0] = v0;
-                    p4[1] = v1;
+            if (d.info & kWrite) {
+                // the query token's K/V: into the pool at position L - 1 and
+                // over the stale row of this stage
+                const int off = valid - 1;
+                if (lane < 2 * CPR) {
+                    const bool isv = lane >= CPR;
+                    const int c = isv ? lane - CPR : lane;
+                    uint16_t *cache = static_cast<uint16_t *>(const_cast<void *>(isv ? a.v_cache : a.k_cache));
+                    *reinterpret_cast<uint4 *>(cache + (((int64_t)d.phys * Hkv + d.h) * 16 + off) * D + c * 8) = kvn;
+                    const uint32_t dst = (isv ? vb : kb) + tile_off(off, c);
+                    asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(dst), "r"(kvn.x), "r"(kvn.y),
+                                 "r"(kvn.z), "r"(kvn.w)
+                                 : "memory");
                 }
-                if (lr == 0) ml_part[slot] = make_float2(st.m[c], st.l[c]);
+            }
+            if (valid < 16) {
+                // keys past the context: p = 0, but their V rows may hold
+                // anything (0 * NaN = NaN in the MMA), so clear them
+                for (int i = lane; i < (16 - max(valid, 0)) * CPR; i += 32) {
+                    const int row = max(valid, 0) + i / CPR, c = i % CPR;
+                    asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};" ::"r"(vb + tile_off(row, c)), "r"(0)
+                                 : "memory");
+                }
+            }
+            if (u + 1 < nu) {
+                // a piece that starts next and ends with the query token's
+                // row: its new K/V in flight from now on
+                const SlotDesc d1 = mydesc[s + 1 == S ? 0 : s + 1];
+                if (d1.info & kWriteSoon) load_new(d1);
+            }
+            __syncwarp();
+            attend_block<D>(st, kb, vb, qf, lane, valid, a.scale_log2);
+            if (d.info & kLast) {
+                // row-group reduction of the thread-partial sums, then the
+                // unnormalised partial of this piece
+                float l0 = st.l[0], l1 = st.l[1];
+#pragma unroll
+                for (int off = 4; off < 32; off <<= 1) {
+                    l0 += __shfl_xor_sync(0xffffffffu, l0, off);
+                    l1 += __shfl_xor_sync(0xffffffffu, l1, off);
+                }
+#pragma unroll
+                for (int c = 0; c < 2; ++c) {
+                    const int hd = 2 * (lane & 3) + c;
+                    if (hd < g) {
+                        const int64_t slot = ((int64_t)d.r * Hq + d.h * g + hd) * lay.parts_per_head + d.part;
+                        float *dst = o_part + slot * D + (lane >> 2);
+#pragma unroll
+                        for (int mt = 0; mt < D / 16; ++mt) {
+                            dst[16 * mt] = st.o[mt][c];
+                            dst[16 * mt + 8] = st.o[mt][2 + c];
+                        }
+                        if ((lane >> 2) == 0) ml_part[slot] = make_float2(st.m[c], c ? l1 : l0);
+                    }
+                }
+            }
+            __syncwarp();
+            if (u + S < nu) produce(s);
+            if (++s == S) {
+                s = 0;
+                phase ^= 1u;
             }
         }
-        if (x == seg_off && lane == 0) {
-            // the segment's part counts for the combine: private pieces in the
-            // low half, the prefix pass's partials of its group in the high one
-            const int32_t n_priv = (int32_t)((seg_off + n - 1) / per - seg_off / per + 1);
-            const int32_t n_pre = lay.prefix_parts > 0 && a.num_groups > 0
-                                      ? min((sh + lay.prefix_blocks_per_part - 1) / lay.prefix_blocks_per_part,
-                                            lay.prefix_parts)
-                                      : 0;
-            nparts[(int64_t)r * Hkv + h] = n_priv | (n_pre << 16);
+        if (u < nu) {
+            // a wait ran out: latch it, then let this warp's copies still in
+            // flight (units u .. u + S - 1) land before the CTA exits
+            if (lane == 0) {
+                latch_error(a.err, kDevTimeout);
+                int quiet = 0;
+                for (int64_t v = u; v < nu && v < u + S; ++v) {
+                    const int sv = (int)(v % S);
+                    mbar_wait(mybar + 8 * sv, (uint32_t)((v / S) & 1), &quiet, kDrainLimitNs);
+                }
+            }
+            __syncwarp();
         }
-        x = piece_end;
-      }
-    }
-    // the last warp out leaves both counters at zero for the next call
-    if (lane == 0 && atomicAdd(a.sched + 1, 1) == (int)(gridDim.x * kWarps) - 1) {
-        atomicExch(a.sched, 0);
-        atomicExch(a.sched + 1, 0);
     }
     if (after_prefix) pdl_wait();
 }
@@ -481,46 +649,71 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(DecodeArgs a, Decod
 
 }  // namespace
 
+namespace {
+
+// Shared memory of the split pass for `stages` ring stages.
+size_t split_smem_bytes(int32_t R, int32_t d, int stages) {
+    const size_t slot = 2 * (size_t)(d / 64) * 2048 + 8 * (size_t)d * 2;   // K/V tiles + Q area
+    return 1024 + (size_t)kWarps * stages * (slot + sizeof(SlotDesc) + 8) + 4 * ((size_t)R + 1);
+}
+
+}  // namespace
+
 DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_t max_blocks,
                            int32_t num_groups, int32_t max_group_blocks, int32_t max_group_members,
                            int32_t num_sms) {
     DecodeLayout L{};
     L.R = R; L.Hq = Hq; L.Hkv = Hkv; L.d = d; L.g = Hq / Hkv;
     L.sms = num_sms > 0 ? num_sms : 148;
+    const int sms = L.sms;
     L.prefix_blocks_per_part = 8;
     L.prefix_parts = 0;
+    L.prefix_ctas = 0;
+    L.prefix_early = 0;
+    // the private split pass streams about kSplitGBsPerSM per SM, together
+    // at most kSplitGBsTotal; its bytes are estimated from the table width
+    // (60 % of the blocks past the longest prefix), which only steers choices
+    constexpr double kSplitGBsPerSM = 50.0, kSplitGBsTotal = 6600.0;
+    const double unit_bytes = 16.0 * d * 2 * 2;   // K + V of one (block, kv head)
+    const double priv_blocks = 0.6 * std::max(1, max_blocks - std::max(0, max_group_blocks));
+    const double split_bytes = (double)R * Hkv * priv_blocks * unit_bytes;
+    auto split_us = [&](int nsm) { return split_bytes / std::min(kSplitGBsTotal, kSplitGBsPerSM * nsm) * 1e-3; };
     if (num_groups > 0 && max_group_blocks > 0 && max_group_members > 0) {
         // Key splits of the prefix pass: one CTA per (group, kv head, member
-        // tile, split), one CTA per SM.  The private split pass runs on the
-        // SMs the prefix pass leaves free (it starts as soon as the prefix
-        // pass has), so a step costs about
-        //   max(prefix critical path, (prefix SM-time + split SM-time) / SMs).
-        // Measured on GB300: a prefix CTA costs about 13 us of fixed work
-        // (set-up, Q tile, pipeline fill, partial writes) plus 2.1 us per key
-        // tile; the split pass streams about 41 GB/s per SM.  The private
-        // work is estimated from the table width (60 % of the blocks past the
-        // longest prefix), which only steers the split count.
+        // tile, split), one CTA per SM.  When its grid leaves at least a
+        // quarter of the SMs free, the split pass runs beside it on those
+        // SMs and a step costs about max(prefix critical path, split time on
+        // the free SMs); otherwise the two run one after the other.
+        // Measured on GB300: a prefix CTA costs about 16 us of fixed work
+        // (set-up, Q tile, pipeline fill, partial writes, with the split pass
+        // loading HBM beside it) plus 2.1 us per key tile.
         const int per_item = 2 * (128 / L.g);   // members per work item (two 128-row tiles)
         const int64_t tiles = (int64_t)num_groups * Hkv * ((max_group_members + per_item - 1) / per_item);
-        const int sms = num_sms > 0 ? num_sms : 148;
         const int key_tiles = (max_group_blocks + 7) / 8;
-        const double unit_bytes = 16.0 * d * 2 * 2;   // K + V of one (block, kv head)
-        const double priv_blocks = 0.6 * std::max(1, max_blocks - max_group_blocks);
-        const double split_sm_us = (double)R * Hkv * priv_blocks * unit_bytes / 41e3;
         int best = 1;
         double best_t = 1e300;
         for (int sp = 1; sp <= kMaxPrefixParts && sp <= key_tiles; ++sp) {
             const int per = (key_tiles + sp - 1) / sp;
             const int64_t ctas = tiles * sp;
-            const double cta_us = 13.0 + 2.1 * per;
+            const double cta_us = 16.0 + 2.1 * per;
             const double crit = (double)((ctas + sms - 1) / sms) * cta_us;
-            const double t = std::max(crit, (ctas * cta_us + split_sm_us) / sms);
+            const double t = (4 * ctas <= 3 * (int64_t)sms) ? std::max(crit, split_us(sms - (int)ctas))
+                                                           : crit + split_us(sms);
             if (t < best_t - 1e-9) { best_t = t; best = sp; }
         }
         const int per_tiles = (key_tiles + best - 1) / best;
         L.prefix_blocks_per_part = per_tiles * 8;
         L.prefix_parts = (max_group_blocks + L.prefix_blocks_per_part - 1) / L.prefix_blocks_per_part;
+        L.prefix_ctas = tiles * L.prefix_parts;
+        L.prefix_early = (4 * L.prefix_ctas <= 3 * (int64_t)sms) ? 1 : 0;
     }
+    L.split_grid = L.prefix_early ? sms - (int32_t)L.prefix_ctas : sms;
+    // as many ring stages as fit (the plan takes 4 bytes per request)
+    L.stages = 2;
+    const int max_stages = d == 64 ? 4 : 3;
+    for (int st = max_stages; st > 2; --st)
+        if (split_smem_bytes(R, d, st) <= kMaxSmemPerBlock) { L.stages = st; break; }
+    L.split_smem = split_smem_bytes(R, d, L.stages);
     L.parts_per_head = L.prefix_parts + kMaxPrivateParts;
     const size_t slots = (size_t)R * Hq * L.parts_per_head;
     auto up = [](size_t x) { return (x + 255) & ~(size_t)255; };
@@ -532,41 +725,41 @@ DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_
 }
 
 template <int D>
-static cudaError_t launch_decode_t(const DecodeLayout &L, const DecodeArgs &a, int num_sms,
-                                   int32_t num_blocks_pool, cudaStream_t stream, Tracer *tr) {
-    if (L.prefix_parts > 0 && a.num_groups > 0) {
+static cudaError_t launch_decode_t(const DecodeLayout &L, const DecodeArgs &a, int32_t num_blocks_pool,
+                                   cudaStream_t stream, Tracer *tr) {
+    const bool prefix = L.prefix_parts > 0 && a.num_groups > 0;
+    if (prefix) {
         cudaError_t e = launch_decode_prefix(L, a, num_blocks_pool, stream, tr);
         if (e != cudaSuccess) return e;
     }
-    const size_t smem = (size_t)(L.R + 1) * sizeof(int32_t);
-    static size_t attr_bytes = 0;
-    if (smem > 48 * 1024 && smem > attr_bytes) {
-        cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<D>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    static SmemLimit limit;
+    {
+        cudaError_t e = limit.ensure(reinterpret_cast<const void *>(decode_split_kernel<D>), (int)L.split_smem);
         if (e != cudaSuccess) return e;
-        attr_bytes = smem;
     }
     if (tr) tr->begin(kKernelDecodeSplit, stream);
-    const int32_t after_prefix = (L.prefix_parts > 0 && a.num_groups > 0) ? 1 : 0;
-    cudaError_t e = launch_pdl(decode_split_kernel<D>, dim3(num_sms), dim3(kThreads), smem, stream,
-                               a, L, num_blocks_pool, after_prefix);
+    // the split pass runs beside an early-triggering prefix pass on the SMs
+    // it leaves free, after a late-triggering one on all of them
+    const int grid = prefix ? L.split_grid : L.sms;
+    cudaError_t e = launch_pdl(decode_split_kernel<D>, dim3(grid), dim3(kThreads), L.split_smem, stream,
+                               *a.tmap_k, *a.tmap_v, a, L, num_blocks_pool, prefix ? 1 : 0);
     if (tr) tr->end(kKernelDecodeSplit, stream);
     if (e != cudaSuccess) return e;
     // four warps per CTA: small batches spread over more SMs
     const int64_t items = (int64_t)L.R * L.Hkv;
-    const int64_t grid = (items + 3) / 4;
-    if (grid > 0x7fffffff) return cudaErrorInvalidConfiguration;
+    const int64_t cgrid = (items + 3) / 4;
+    if (cgrid > 0x7fffffff) return cudaErrorInvalidConfiguration;
     if (tr) tr->begin(kKernelDecodeCombine, stream);
-    e = L.g <= 4 ? launch_pdl(decode_combine_kernel<D, 4>, dim3((unsigned)grid), dim3(128), 0, stream, a, L)
-                 : launch_pdl(decode_combine_kernel<D, 8>, dim3((unsigned)grid), dim3(128), 0, stream, a, L);
+    e = L.g <= 4 ? launch_pdl(decode_combine_kernel<D, 4>, dim3((unsigned)cgrid), dim3(128), 0, stream, a, L)
+                 : launch_pdl(decode_combine_kernel<D, 8>, dim3((unsigned)cgrid), dim3(128), 0, stream, a, L);
     if (tr) tr->end(kKernelDecodeCombine, stream);
     return e;
 }
 
-cudaError_t launch_decode(const DecodeLayout &L, const DecodeArgs &a, int num_sms,
-                          int32_t num_blocks_pool, cudaStream_t stream, Tracer *tr) {
-    if (L.d == 128) return launch_decode_t<128>(L, a, num_sms, num_blocks_pool, stream, tr);
-    return launch_decode_t<64>(L, a, num_sms, num_blocks_pool, stream, tr);
+cudaError_t launch_decode(const DecodeLayout &L, const DecodeArgs &a, int32_t num_blocks_pool,
+                          cudaStream_t stream, Tracer *tr) {
+    if (L.d == 128) return launch_decode_t<128>(L, a, num_blocks_pool, stream, tr);
+    return launch_decode_t<64>(L, a, num_blocks_pool, stream, tr);
 }
 
 }  // namespace pkv

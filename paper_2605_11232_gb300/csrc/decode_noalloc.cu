@@ -23,7 +23,7 @@ namespace {
 // Largest workspace this entry point can serve.  Every GPU that loads the
 // library holds this array until the process exits.
 constexpr size_t kScratchBytes = size_t(64) << 20;
-constexpr int kMaxDevices = 64;
+using pkv::kMaxDevices;
 
 __device__ __align__(256) unsigned char g_decode_scratch[kScratchBytes];
 
@@ -51,16 +51,20 @@ extern "C" int paged_attn_decode_noalloc(pkv_pool_t pool, const void *q, void *o
                  need, kScratchBytes);
         return pkv::set_last_error(PKV_ERR_WORKSPACE, msg);
     }
-    // the device that owns the caller's buffers
+    // the kernels run on the pool's device: the scratch address must be that
+    // device's, and q must live there too
+    int dev = -1;
+    rc = pkv::pool_device(pool, &dev);
+    if (rc != PKV_OK) return rc;
+    if (dev < 0 || dev >= kMaxDevices)
+        return pkv::set_last_error(PKV_ERR_INVALID_ARG, "paged_attn_decode_noalloc: pool device out of range");
     cudaPointerAttributes attr;
     cudaError_t e = cudaPointerGetAttributes(&attr, q);
-    if (e != cudaSuccess || attr.type != cudaMemoryTypeDevice || attr.device < 0 ||
-        attr.device >= kMaxDevices) {
+    if (e != cudaSuccess || attr.type != cudaMemoryTypeDevice || attr.device != dev) {
         cudaGetLastError();
         return pkv::set_last_error(PKV_ERR_INVALID_ARG,
-                                   "paged_attn_decode_noalloc: q is not device memory");
+                                   "paged_attn_decode_noalloc: q is not device memory of the pool's device");
     }
-    const int dev = attr.device;
     void *scratch = nullptr;
     {
         // one-time set-up on this device, with the device current: the host

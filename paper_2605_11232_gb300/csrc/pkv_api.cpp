@@ -79,7 +79,7 @@ struct pkv_pool {
     void *v_cache = nullptr;
     std::vector<int32_t> refcnt;     // 0 = free
     std::vector<int32_t> free_list;  // back() is handed out next
-    int *d_err = nullptr;            // device words: [0] error, [1..2] decode split scheduling
+    int *d_err = nullptr;            // device error word (latched by the kernels)
     int device = -1;
     int num_sms = 0;
     bool tmaps_ready = false;
@@ -174,10 +174,32 @@ int build_tmaps(pkv_pool_t pool) {
 }  // namespace
 
 namespace pkv {
+cudaError_t SmemLimit::ensure(const void *func, int need) {
+    if (need <= 48 * 1024) return cudaSuccess;   // no opt-in below the default limit
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    if (bytes[dev].load(std::memory_order_acquire) >= need) return cudaSuccess;
+    std::lock_guard<std::mutex> lock(mu);
+    const int have = bytes[dev].load(std::memory_order_relaxed);
+    if (have >= need) return cudaSuccess;
+    e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, need);
+    if (e == cudaSuccess) bytes[dev].store(need, std::memory_order_release);
+    return e;
+}
+
 // Record a failure message for pkv_last_error() from another translation unit.
 int set_last_error(int code, const char *msg) {
     g_last_error = msg ? msg : "";
     return code;
+}
+
+int pool_device(pkv_pool_t pool, int *dev) {
+    int rc = check_kernel_pool(pool);
+    if (rc != PKV_OK) return rc;
+    *dev = pool->device;
+    return PKV_OK;
 }
 
 int pool_device_error_word(pkv_pool_t pool, int **err) {
@@ -225,10 +247,9 @@ int kv_pool_create(const pkv_pool_desc *desc, void *k_cache, void *v_cache, pkv_
     if (k_cache) {
         cudaError_t e = cudaGetDevice(&p->device);
         if (e == cudaSuccess) e = cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount, p->device);
-        // the error word, then the decode split pass's work and done
-        // counters (zero between calls: the pass's last warp resets them)
-        if (e == cudaSuccess) e = cudaMalloc(&p->d_err, 4 * sizeof(int));
-        if (e == cudaSuccess) e = cudaMemset(p->d_err, 0, 4 * sizeof(int));
+        // the device error word
+        if (e == cudaSuccess) e = cudaMalloc(&p->d_err, sizeof(int));
+        if (e == cudaSuccess) e = cudaMemset(p->d_err, 0, sizeof(int));
         if (e != cudaSuccess) {
             if (p->d_err) cudaFree(p->d_err);
             delete p;
@@ -339,7 +360,9 @@ int kv_slot_mapping(pkv_pool_t pool, const int32_t *block_table, int32_t max_blo
             const int32_t blk = block_table[(int64_t)r * max_blocks + p / 16];
             if (blk < 0) return fail(PKV_ERR_INVALID_ARG, "request %d: no block for position %lld", r, (long long)p);
             if (pool) {
-                if (blk >= pool->desc.num_blocks || pool->refcnt[blk] == 0)
+                if (blk >= pool->desc.num_blocks)
+                    return fail(PKV_ERR_INVALID_ARG, "request %d: block id %d is outside the pool", r, blk);
+                if (pool->refcnt[blk] == 0)
                     return fail(PKV_ERR_REFCOUNT, "request %d: block %d is not allocated", r, blk);
                 if (pool->refcnt[blk] > 1)
                     return fail(PKV_ERR_SHARED_BLOCK_WRITE,
@@ -371,7 +394,7 @@ int pkv_check_block_table(pkv_pool_t pool, const int32_t *block_table, int32_t m
             for (int64_t j = 0; j < nblk && rc == PKV_OK; ++j) {
                 const int32_t id = row[j];
                 if (id < 0 || id >= pool->desc.num_blocks)
-                    rc = fail(PKV_ERR_REFCOUNT, "request %d: entry %lld holds block id %d, outside the pool",
+                    rc = fail(PKV_ERR_INVALID_ARG, "request %d: entry %lld holds block id %d, outside the pool",
                               r, (long long)j, id);
                 else if (pool->refcnt[id] == 0)
                     rc = fail(PKV_ERR_REFCOUNT, "request %d: entry %lld holds free block %d", r,
@@ -419,6 +442,9 @@ int paged_attn_prefill(pkv_pool_t pool, const void *q, void *out, float *lse,
         return fail(PKV_ERR_INVALID_ARG, "num_q_heads must be a positive multiple of num_kv_heads");
     if (num_q_heads / d.num_kv_heads > 128)
         return fail(PKV_ERR_UNSUPPORTED, "more than 128 q heads per kv head");
+    if (max_blocks > pkv::kPrefillMaxBlocks)
+        return fail(PKV_ERR_UNSUPPORTED, "table width %d: prefill supports contexts up to %d blocks (%d tokens)",
+                    max_blocks, pkv::kPrefillMaxBlocks, 16 * pkv::kPrefillMaxBlocks);
     if (!(scale > 0.f) || !std::isfinite(scale)) return fail(PKV_ERR_INVALID_ARG, "bad scale");
     if (num_requests == 0 || max_seqlen_q == 0) return ok();
     if (!q || !out || !cu_seqlens_q || !context_lens || !block_table)
@@ -463,8 +489,8 @@ namespace {
 // Every host-side check of paged_attn_decode, then its layout and kernel
 // arguments (and the pool's TMA descriptors when the prefix pass runs);
 // nothing is enqueued.  *empty: no request, nothing to launch.
-int prepare_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
-                   const int32_t *context_lens, const int32_t *block_table, int32_t max_blocks,
+int prepare_decode(pkv_pool_t pool, const void *q, const void *k_new, const void *v_new, void *out,
+                   float *lse, const int32_t *context_lens, const int32_t *block_table, int32_t max_blocks,
                    int32_t num_requests, int32_t num_q_heads, float scale,
                    const pkv_prefix_groups *groups, void *workspace, size_t workspace_bytes,
                    pkv::DecodeLayout *L_out, pkv::DecodeArgs *a_out, bool *empty) {
@@ -483,6 +509,9 @@ int prepare_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
     if (*empty) return ok();
     if (!q || !out || !context_lens || !block_table) return fail(PKV_ERR_INVALID_ARG, "NULL buffer");
     if (!aligned16(q) || !aligned16(out)) return fail(PKV_ERR_INVALID_ARG, "misaligned q/out");
+    if ((k_new == nullptr) != (v_new == nullptr)) return fail(PKV_ERR_INVALID_ARG, "give both k_new and v_new");
+    if (k_new && (!aligned16(k_new) || !aligned16(v_new)))
+        return fail(PKV_ERR_INVALID_ARG, "misaligned k_new/v_new");
     int32_t G = 0, mgb = 0, mgm = 0;
     if (groups && groups->num_groups > 0) {
         G = groups->num_groups;
@@ -502,7 +531,7 @@ int prepare_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
     if (reinterpret_cast<uintptr_t>(workspace) & 255)
         return fail(PKV_ERR_WORKSPACE, "workspace must be 256-byte aligned");
     if ((rc = set_device(pool)) != PKV_OK) return rc;
-    if (L.prefix_parts > 0 && (rc = build_tmaps(pool)) != PKV_OK) return rc;
+    if ((rc = build_tmaps(pool)) != PKV_OK) return rc;
     pkv::DecodeArgs &a = *a_out;
     a = pkv::DecodeArgs{};
     a.q = q; a.out = out; a.lse = lse;
@@ -517,9 +546,10 @@ int prepare_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
     }
     a.ws = workspace;
     a.err = pool->d_err;
-    a.sched = pool->d_err + 1;
     a.tmap_k = &pool->tmap_k;
     a.tmap_v = &pool->tmap_v;
+    a.k_new = k_new;
+    a.v_new = v_new;
     return ok();
 }
 
@@ -535,12 +565,32 @@ int paged_attn_decode(pkv_pool_t pool, const void *q, void *out, float *lse,
     pkv::DecodeLayout L{};
     pkv::DecodeArgs a{};
     bool empty = true;
-    const int rc = prepare_decode(pool, q, out, lse, context_lens, block_table, max_blocks, num_requests,
-                                  num_q_heads, scale, groups, workspace, workspace_bytes, &L, &a, &empty);
+    const int rc = prepare_decode(pool, q, nullptr, nullptr, out, lse, context_lens, block_table, max_blocks,
+                                  num_requests, num_q_heads, scale, groups, workspace, workspace_bytes, &L, &a,
+                                  &empty);
     if (rc != PKV_OK || empty) return rc;
-    cudaError_t e = pkv::launch_decode(L, a, pool->num_sms, pool->desc.num_blocks,
-                                       static_cast<cudaStream_t>(stream), pool->tracer);
+    cudaError_t e = pkv::launch_decode(L, a, pool->desc.num_blocks, static_cast<cudaStream_t>(stream),
+                                       pool->tracer);
     if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode launch");
+    return ok();
+}
+
+int paged_attn_decode_append(pkv_pool_t pool, const void *q, const void *k_new, const void *v_new,
+                             void *out, float *lse, const int32_t *context_lens,
+                             const int32_t *block_table, int32_t max_blocks, int32_t num_requests,
+                             int32_t num_q_heads, float scale, const pkv_prefix_groups *groups,
+                             void *workspace, size_t workspace_bytes, pkv_stream_t stream) {
+    if (num_requests > 0 && (!k_new || !v_new)) return fail(PKV_ERR_INVALID_ARG, "NULL k_new/v_new");
+    pkv::DecodeLayout L{};
+    pkv::DecodeArgs a{};
+    bool empty = true;
+    const int rc = prepare_decode(pool, q, k_new, v_new, out, lse, context_lens, block_table, max_blocks,
+                                  num_requests, num_q_heads, scale, groups, workspace, workspace_bytes, &L, &a,
+                                  &empty);
+    if (rc != PKV_OK || empty) return rc;
+    cudaError_t e = pkv::launch_decode(L, a, pool->desc.num_blocks, static_cast<cudaStream_t>(stream),
+                                       pool->tracer);
+    if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode_append launch");
     return ok();
 }
 
@@ -576,7 +626,7 @@ int paged_attn_decode_step(pkv_pool_t pool, const void *host_in, void *dev_in,
     pkv::DecodeLayout L{};
     pkv::DecodeArgs a{};
     bool empty = true;
-    rc = prepare_decode(pool, din + layout->q, out, lse,
+    rc = prepare_decode(pool, din + layout->q, nullptr, nullptr, out, lse,
                         reinterpret_cast<const int32_t *>(din + layout->context_lens), block_table,
                         max_blocks, num_requests, num_q_heads, scale, groups, workspace, workspace_bytes,
                         &L, &a, &empty);
@@ -594,7 +644,7 @@ int paged_attn_decode_step(pkv_pool_t pool, const void *host_in, void *dev_in,
                         stream);
     if (rc != PKV_OK) return rc;
     if (!empty) {
-        e = pkv::launch_decode(L, a, pool->num_sms, d.num_blocks, st, pool->tracer);
+        e = pkv::launch_decode(L, a, d.num_blocks, st, pool->tracer);
         if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode_step launch");
     }
     if (done_event) {

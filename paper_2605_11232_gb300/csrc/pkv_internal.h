@@ -6,6 +6,9 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+#include <mutex>
+
 struct pkv_pool;   // the pool handle's struct (include/pkv.h: pkv_pool_t)
 
 namespace pkv {
@@ -50,8 +53,28 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
 
+// A kernel's dynamic shared-memory limit (cudaFuncAttributeMaxDynamicSharedMemorySize)
+// is a per-device setting.  One SmemLimit per kernel instantiation records,
+// per device, the largest limit set so far; ensure() raises it on the current
+// device when a launch needs more.  Thread-safe: the limit only grows, under
+// the lock, so two threads launching on one device never lower each other's.
+constexpr int kMaxDevices = 64;
+struct SmemLimit {
+    std::atomic<int> bytes[kMaxDevices] = {};
+    std::mutex mu;
+    cudaError_t ensure(const void *func, int need);
+};
+
+// Largest table width paged_attn_prefill accepts: a work item's block ids are
+// staged in shared memory, at most kPrefillMaxBlocks of them (32768 keys).
+constexpr int kPrefillMaxBlocks = 2048;
+
 // Set the thread's pkv_last_error() message; returns code.
 int set_last_error(int code, const char *msg);
+
+// The device a pool's caches live on (the one its kernels launch on), after
+// checking that the pool has device caches; PKV_OK or an error code.
+int pool_device(::pkv_pool *pool, int *dev);
 
 // The pool's device error word, after checking that the pool has device
 // caches and making its device current; PKV_OK or an error code.
@@ -73,11 +96,18 @@ constexpr int kMaxPrivateParts = 16;
 constexpr int kMaxPrefixParts = 16;   // parts_per_head <= 32: one part per combine lane
 constexpr int kMinBlocksPerPiece = 4;
 
+constexpr size_t kMaxSmemPerBlock = 227 * 1024;   // opt-in dynamic shared memory per CTA
+
 struct DecodeLayout {
     int32_t R, Hq, Hkv, d, g;
     int32_t sms;                 // SMs of the device the layout was made for
     int32_t prefix_parts;        // prefix-pass part slots per head (0 without groups)
     int32_t prefix_blocks_per_part;
+    int64_t prefix_ctas;         // CTAs of the prefix pass (0 without groups)
+    int32_t prefix_early;        // the prefix pass lets the split pass start beside it
+    int32_t split_grid;          // split-pass CTAs beside an early prefix pass
+    int32_t stages;              // ring stages per warp of the split pass
+    size_t split_smem;           // dynamic shared memory of the split pass
     int32_t parts_per_head;      // prefix_parts + kMaxPrivateParts
     // byte offsets inside the workspace
     size_t off_o;                // float [R*Hq*parts][d]
@@ -113,13 +143,16 @@ struct DecodeArgs {
     const int32_t *group_of_req;
     void *ws;
     int *err;
-    int *sched;                  // [0] next chunk, [1] warps done (the split pass)
-    const CUtensorMap *tmap_k;   // needed by the shared-prefix pass
+    const CUtensorMap *tmap_k;   // TMA descriptors of the pool's caches
     const CUtensorMap *tmap_v;
+    // the query tokens' own K/V, bf16 [R][Hkv][d], stored at position L - 1
+    // by the split pass (paged_attn_decode_append); null: already in the cache
+    const void *k_new;
+    const void *v_new;
 };
 
-cudaError_t launch_decode(const DecodeLayout &L, const DecodeArgs &a, int num_sms,
-                          int32_t num_blocks_pool, cudaStream_t stream, Tracer *tr);
+cudaError_t launch_decode(const DecodeLayout &L, const DecodeArgs &a, int32_t num_blocks_pool,
+                          cudaStream_t stream, Tracer *tr);
 
 struct PrefillArgs {
     const void *q;

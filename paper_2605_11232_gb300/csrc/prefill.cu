@@ -52,7 +52,7 @@ constexpr int kKeys = 128;            // keys per K/V tile (N of Q.K^T)
 constexpr uint32_t kTmemCols = 512;   // S_A [0,128) S_B [128,256) O_A [256,384) O_B [384,512)
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr uint64_t kDrainLimitNs = 200000000ull;
-constexpr int kMaxItemBlocks = 2048;  // keys of one work item <= 32768
+constexpr int kMaxItemBlocks = kPrefillMaxBlocks;  // keys of one work item <= 32768
 template <int D>
 struct Layout {
     static constexpr int kHalves = D / 64;            // 64-element (128-byte) column halves
@@ -602,16 +602,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 template <int D, bool PREFIX>
 static cudaError_t launch_tile_kernel(dim3 grid, const CUtensorMap &tk, const CUtensorMap &tv,
                                       const KernelParams &p, cudaStream_t stream) {
-    static bool attr = false;
     // the d = 64 tiles are smaller; ask for the d = 128 footprint anyway so
     // one CTA owns an SM (its 512 TMEM columns never wait on a neighbour)
-    if (!attr) {
-        cudaError_t e = cudaFuncSetAttribute(attn_tile_kernel<D, PREFIX>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             Layout<128>::kDynSmem);
-        if (e != cudaSuccess) return e;
-        attr = true;
-    }
+    static SmemLimit limit;
+    cudaError_t e = limit.ensure(reinterpret_cast<const void *>(attn_tile_kernel<D, PREFIX>),
+                                 Layout<128>::kDynSmem);
+    if (e != cudaSuccess) return e;
     return launch_pdl(attn_tile_kernel<D, PREFIX>, grid, dim3(kThreads), Layout<128>::kDynSmem, stream,
                       tk, tv, p);
 }
@@ -667,8 +663,7 @@ cudaError_t launch_decode_prefix(const DecodeLayout &L, const DecodeArgs &a,
     // at least a quarter of the device.  A pass that fills nearly every SM
     // keeps its successor until it exits: starting the split pass early
     // there measured much slower (l70b decode 345 -> 433 us per step).
-    const int64_t ctas = (int64_t)grid.x * grid.y * grid.z;
-    p.early_trigger = (4 * ctas <= 3 * (int64_t)L.sms) ? 1 : 0;
+    p.early_trigger = L.prefix_early;
     if (tr) tr->begin(kKernelDecodePrefix, stream);
     cudaError_t e = L.d == 128 ? launch_tile_kernel<128, true>(grid, *a.tmap_k, *a.tmap_v, p, stream)
                                : launch_tile_kernel<64, true>(grid, *a.tmap_k, *a.tmap_v, p, stream);

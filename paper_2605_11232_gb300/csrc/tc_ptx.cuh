@@ -176,8 +176,6 @@ __device__ __forceinline__ void tmem_wait_st() {
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
-// ---- register rebalancing between warpgroups ---------------------------------
-
 // ---- tcgen05.mma ----------------------------------------------------------------
 
 // Shared-memory matrix descriptor, 128-byte swizzle.  Fields: start address,

@@ -38,7 +38,7 @@ EXPORTS = [
     "kv_pool_create", "kv_pool_destroy", "kv_pool_alloc", "kv_pool_retain", "kv_pool_release",
     "kv_pool_refcount", "kv_pool_num_free", "kv_pool_alloc_sequence", "kv_slot_mapping",
     "kv_cache_write", "paged_attn_prefill", "paged_attn_decode_workspace_size",
-    "paged_attn_decode", "paged_attn_decode_noalloc", "paged_attn_decode_step", "pkv_trace_enable",
+    "paged_attn_decode", "paged_attn_decode_append", "paged_attn_decode_noalloc", "paged_attn_decode_step", "pkv_trace_enable",
     "pkv_trace_read", "pkv_check_device_errors", "pkv_last_error", "pkv_prefix_cache_create",
     "pkv_prefix_cache_destroy", "pkv_prefix_cache_match", "pkv_prefix_cache_insert",
     "pkv_prefix_cache_evict", "pkv_prefix_cache_size", "pkv_prefix_groups_build",
@@ -109,6 +109,8 @@ def load(path: str | None = None):
                                              ctypes.POINTER(sz)],
         "paged_attn_decode": [V, V, V, V, V, V, i32, i32, i32, f32,
                               ctypes.POINTER(PrefixGroups), V, sz, V],
+        "paged_attn_decode_append": [V, V, V, V, V, V, V, V, i32, i32, i32, f32,
+                                     ctypes.POINTER(PrefixGroups), V, sz, V],
         "pkv_check_device_errors": [V, V, P],
         "paged_attn_decode_noalloc": [V, V, V, V, V, V, i32, i32, i32, f32,
                                       ctypes.POINTER(PrefixGroups), V],
@@ -382,6 +384,28 @@ def paged_attn_decode(pool, q, out, lse, context_lens, block_table, scale: float
     _check(load().paged_attn_decode(
         pool, _dptr(q), _dptr(out), _dptr(lse), _dptr(context_lens), _dptr(block_table),
         int(block_table.shape[1]), int(context_lens.shape[0]), int(q.shape[1]), float(scale),
+        ctypes.byref(groups) if groups is not None else None, _dptr(workspace),
+        int(workspace.numel() * workspace.element_size()) if workspace is not None else 0,
+        _stream(stream)))
+
+
+def paged_attn_decode_append(pool, q, k_new, v_new, out, lse, context_lens, block_table, scale: float,
+                             groups, workspace, stream=None):
+    """paged_attn_decode with the query tokens' own K/V (bf16 [R][Hkv][d])
+    stored into the pool by the decode kernels."""
+    import torch
+    R = int(context_lens.shape[0])
+    _check_attn_args(pool, q, out, lse, context_lens, block_table, R)
+    geo = _pool_geometry(pool)
+    for name, t in (("k_new", k_new), ("v_new", v_new)):
+        ts = _check_tensor(name, t, torch.bfloat16, 3)
+        _need(ts[0] >= R, lambda: f"{name} has {ts[0]} rows, {R} needed")
+        if geo is not None:
+            _need(ts[1] == geo[1] and ts[2] == geo[2],
+                  lambda: f"{name} rows must be [{geo[1]}][{geo[2]}], got {list(ts[1:])}")
+    _check(load().paged_attn_decode_append(
+        pool, _dptr(q), _dptr(k_new), _dptr(v_new), _dptr(out), _dptr(lse), _dptr(context_lens),
+        _dptr(block_table), int(block_table.shape[1]), R, int(q.shape[1]), float(scale),
         ctypes.byref(groups) if groups is not None else None, _dptr(workspace),
         int(workspace.numel() * workspace.element_size()) if workspace is not None else 0,
         _stream(stream)))

@@ -35,6 +35,27 @@ def run_decode(b, use_groups=False, with_lse=True):
     return out, lse
 
 
+def run_decode_append(b, use_groups=False, with_lse=True):
+    """The decode subset's cache write and attention in one call
+    (paged_attn_decode_append); the prefill subset's new tokens, if any, by
+    kv_cache_write, so the pool ends as after run_decode."""
+    w = b.w
+    Rd = b.dec.stop - b.dec.start
+    rows_p = B.new_token_rows(w, b.pre)
+    if rows_p.stop > rows_p.start:
+        pkv.kv_cache_write(b.pool, b.k_new[rows_p], b.v_new[rows_p], b.slots[rows_p])
+    out = torch.empty((Rd, w.num_q_heads, w.head_dim), dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty((Rd, w.num_q_heads), dtype=torch.float32, device="cuda") if with_lse else None
+    ws = B.decode_workspace(b, use_groups)
+    B.run_decode_append(b, out, lse, ws, use_groups)
+    assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
+    return out, lse
+
+
+def _bits(t):
+    return t.view(torch.int16)
+
+
 def compare(b, out, lse, reqs, threads=8):
     w = b.w
     errs, lerrs = [], []
@@ -71,38 +92,102 @@ def test_decode_matches_oracle(name, scale, groups):
     b.close()
 
 
+@pytest.mark.parametrize("groups", [True, False])
 @pytest.mark.parametrize("name", ["l8b_decode", "qwen_mixed", "l70b_decode"])
-def test_decode_full_size_sampled_grouped(name):
-    """Full-size batch in the benchmark's launch configuration (grouped prefix
-    pass on): a sample of requests against the oracle, no NaN anywhere."""
+def test_decode_full_size_every_request(name, groups):
+    """Full-size batch in the benchmark's launch configuration (the fused
+    cache write + decode call; groups=True: with the shared-prefix pass):
+    every request's outputs and LSE against the oracle, no NaN anywhere."""
     need_gpu()
     w = make_workload(name)
     b = B.build_batch(w, poison=True)
-    out, lse = run_decode(b, use_groups=True)
+    out, lse = run_decode_append(b, use_groups=groups)
     assert torch.isfinite(out.float()).all()
-    ctx = w.context_lens[b.dec]
-    rng = np.random.default_rng(1)
-    picks = {0, len(ctx) - 1, int(np.argmin(ctx)), int(np.argmax(ctx))}
-    picks |= set(rng.choice(len(ctx), 4, replace=False).tolist())
-    compare(b, out, lse, [b.dec.start + i for i in sorted(picks)], threads=16)
+    compare(b, out, lse, range(b.dec.start, b.dec.stop), threads=16)
     b.close()
 
 
-@pytest.mark.parametrize("name", ["l8b_decode", "qwen_mixed", "l70b_decode"])
-def test_decode_full_size_sampled(name):
-    """Full-size batch, same call as the benchmark; outputs of a sample of
-    requests (first, last, shortest, longest, and random) against the oracle,
-    and no NaN anywhere."""
+@pytest.mark.parametrize("groups", [False, True])
+@pytest.mark.parametrize("name,scale", [
+    ("tiny_decode", 1.0),
+    ("l8b_decode", 0.25),
+    ("qwen_mixed", 0.125),
+    ("l70b_decode", 1 / 32),
+])
+def test_decode_append_equals_write_then_decode(name, scale, groups):
+    """paged_attn_decode_append stores each query token's K/V from inside the
+    decode kernels: its outputs and LSE have the bits of kv_cache_write +
+    paged_attn_decode, and the whole pool afterwards is bit-identical to
+    theirs (NaN-poisoned unused slots included)."""
     need_gpu()
-    w = make_workload(name)
+    w = make_workload(name, scale_requests=scale)
+    b1 = B.build_batch(w, poison=True)
+    o1, l1 = run_decode(b1, use_groups=groups)
+    k1, v1 = b1.k_cache.clone(), b1.v_cache.clone()
+    b1.close()
+    b2 = B.build_batch(w, poison=True)
+    before = _bits(b2.k_cache).clone()
+    o2, l2 = run_decode_append(b2, use_groups=groups)
+    assert torch.equal(o1, o2) and torch.equal(l1, l2)
+    assert torch.equal(_bits(k1), _bits(b2.k_cache)) and torch.equal(_bits(v1), _bits(b2.v_cache))
+    assert not torch.equal(before, _bits(b2.k_cache))   # the call did write the new rows
+    compare(b2, o2, l2, range(b2.dec.start, b2.dec.stop))
+    b2.close()
+
+
+def test_two_pools_two_threads_concurrently():
+    """Two pools on one GPU, each decoded from its own host thread on its own
+    stream, ten times each, concurrently: every output has the bits of the
+    same decode run alone (launch attributes and pool state are per device and
+    per pool, and safe to set up from several threads)."""
+    need_gpu()
+    import threading
+    ws_, refs, bs = [], [], []
+    for name, scale in (("l8b_decode", 0.125), ("qwen_mixed", 0.0625)):
+        w = make_workload(name, scale_requests=scale)
+        b = B.build_batch(w, poison=True)
+        ref, _ = run_decode(b, use_groups=True)
+        bs.append(b)
+        refs.append(ref)
+        ws_.append(B.decode_workspace(b, True))
+    outs = [[torch.empty_like(r) for _ in range(10)] for r in refs]
+    errors = []
+
+    def worker(i):
+        try:
+            s = torch.cuda.Stream()
+            with torch.cuda.stream(s):
+                for k in range(10):
+                    B.run_decode(bs[i], outs[i][k], None, ws_[i], True, stream=s)
+            s.synchronize()
+        except Exception as e:   # reported below
+            errors.append(e)
+
+    threads = [threading.Thread(target=worker, args=(i,)) for i in range(2)]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    torch.cuda.synchronize()
+    assert not errors, errors
+    for i in range(2):
+        assert pkv.pkv_check_device_errors(bs[i].pool) == pkv.PKV_OK
+        for o in outs[i]:
+            assert torch.equal(o, refs[i])
+        bs[i].close()
+
+
+def test_checked_table_then_decode_without_device_errors():
+    """A batch whose rows share refcounted prefix blocks passes the host check
+    of its block tables, and its decode then latches no device error."""
+    need_gpu()
+    w = make_workload("l8b_decode", scale_requests=0.125)
     b = B.build_batch(w, poison=True)
-    out, lse = run_decode(b)
-    assert torch.isfinite(out.float()).all()
-    ctx = w.context_lens[b.dec]
-    rng = np.random.default_rng(0)
-    picks = {0, len(ctx) - 1, int(np.argmin(ctx)), int(np.argmax(ctx))}
-    picks |= set(rng.choice(len(ctx), 4, replace=False).tolist())
-    compare(b, out, lse, [b.dec.start + i for i in sorted(picks)], threads=16)
+    rows = b.table_host[b.dec]
+    assert max(pkv.kv_pool_refcount(b.pool, int(x)) for x in rows[0, :16]) > 1
+    pkv.pkv_check_block_table(b.pool, rows, w.context_lens[b.dec].astype(np.int32))
+    out, lse = run_decode(b, use_groups=True)
+    assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
     b.close()
 
 

@@ -166,10 +166,13 @@ def test_check_block_table_on_the_host():
     for r, row in enumerate(rows):
         table[r, : len(row)] = row
     ctx = np.array([40, 64], np.int32)                  # 3 and 4 blocks
+    # both rows hold the two prefix blocks: reference count 3 (two rows + the
+    # allocation), which the check accepts
+    assert [pkv.kv_pool_refcount(p, int(b)) for b in pre] == [3, 3]
     pkv.pkv_check_block_table(p, table, ctx)            # valid; -1 padding past the context
     table[1, 5] = 999                                   # past request 1's context: not read
     pkv.pkv_check_block_table(p, table, ctx)
-    for r, j, v, code in ((1, 3, 999, pkv.PKV_ERR_REFCOUNT), (0, 2, -1, pkv.PKV_ERR_REFCOUNT),
+    for r, j, v, code in ((1, 3, 999, pkv.PKV_ERR_INVALID_ARG), (0, 2, -1, pkv.PKV_ERR_INVALID_ARG),
                           (1, 0, 31, pkv.PKV_ERR_REFCOUNT)):     # block 31 is free
         bad = table.copy()
         bad[r, j] = v

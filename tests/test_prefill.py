@@ -103,18 +103,45 @@ def test_l8b_prefill_scaled_sampled_rows():
 
 
 @pytest.mark.parametrize("name", ["l8b_prefill", "qwen_mixed"])
-def test_prefill_full_size_sampled(name):
-    """Full-size batch (the benchmark's call); sampled rows of 4 requests vs
-    the oracle and no NaN anywhere in the output."""
+def test_prefill_full_size_every_row(name):
+    """Full-size batch (the benchmark's call): every query row of 8 requests
+    (the first, the last, the middle, the longest cached context and random
+    ones; qwen_mixed has exactly 8) against the oracle, and no NaN anywhere in
+    the output."""
     need_gpu()
     w = make_workload(name)
     b = B.build_batch(w, poison=True)
     out, lse = run_prefill(b)
     assert torch.isfinite(out.float()).all() and torch.isfinite(lse).all()
     reqs = list(range(b.pre.start, b.pre.stop))
-    pick = sorted({reqs[0], reqs[-1], reqs[len(reqs) // 2],
-                   reqs[int(np.argmax(w.cached_lens[b.pre]))]})
-    compare(b, out, lse, pick, rows_per_req=12)
+    pick = {reqs[0], reqs[-1], reqs[len(reqs) // 2], reqs[int(np.argmax(w.cached_lens[b.pre]))]}
+    rng = np.random.default_rng(5)
+    while len(pick) < min(8, len(reqs)):
+        pick.add(int(rng.choice(reqs)))
+    compare(b, out, lse, sorted(pick))
+    b.close()
+
+
+def test_prefill_refuses_tables_wider_than_its_limit():
+    """A work item's block ids are staged in shared memory, 2048 of them at
+    most: a table wider than that is refused on the host (UNSUPPORTED) before
+    any launch."""
+    need_gpu()
+    w = make_workload("tiny")
+    b = B.build_batch(w, poison=True)
+    rows = B.new_token_rows(w, b.pre)
+    wide = torch.full((b.pre.stop - b.pre.start, 2049), -1, dtype=torch.int32, device="cuda")
+    wide[:, : b.table.shape[1]] = b.table[b.pre]
+    out = torch.empty((rows.stop - rows.start, w.num_q_heads, w.head_dim), dtype=torch.bfloat16,
+                      device="cuda")
+    with pytest.raises(pkv.PkvError) as e:
+        pkv.paged_attn_prefill(b.pool, b.q[rows], out, None, b.cu_pre, b.context_lens[b.pre], wide,
+                               b.max_seqlen_pre, w.scale)
+    assert e.value.code == pkv.PKV_ERR_UNSUPPORTED
+    # 2048 columns are accepted
+    pkv.paged_attn_prefill(b.pool, b.q[rows], out, None, b.cu_pre, b.context_lens[b.pre],
+                           wide[:, :2048].contiguous(), b.max_seqlen_pre, w.scale)
+    assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
     b.close()
 
 
