@@ -175,18 +175,18 @@ __device__ __forceinline__ void load_q_smem(uint32_t (&qf)[D / 16][2], uint32_t 
 }
 
 // Block-wide plan: P[r] = sum of the private block counts of requests < r,
-// P[R] = their total; *max_n_out = the largest count.
-__device__ void build_plan(int32_t *P, int32_t R, const int32_t *__restrict__ context_lens,
+// P[R] = their total; Ls[r] = context_lens[r] when Ls is not null;
+// *max_n_out = the largest count.
+__device__ void build_plan(int32_t *P, int32_t *Ls, int32_t R, const int32_t *__restrict__ context_lens,
                            const int32_t *__restrict__ group_of_req,
                            const int32_t *__restrict__ group_blocks, int32_t num_groups,
                            int32_t max_blocks, int32_t *max_n_out, int *err) {
     __shared__ int32_t warp_tot[kWarps];
     __shared__ int32_t warp_max[kWarps];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int per_thread = (R + kThreads - 1) / kThreads;
-    const int r0 = min(R, tid * per_thread), r1 = min(R, r0 + per_thread);
-    int32_t run = 0, mx = 0;
-    for (int r = r0; r < r1; ++r) {
+    // private block counts, request r on thread r % kThreads (independent
+    // loads, in flight together), kept in P for now
+    for (int r = tid; r < R; r += kThreads) {
         const int32_t L = __ldg(context_lens + r);
         int32_t nblk = (L + 15) >> 4;
         if (nblk > max_blocks) {   // context longer than the table row
@@ -202,11 +202,18 @@ __device__ void build_plan(int32_t *P, int32_t R, const int32_t *__restrict__ co
         if (L < 1 || n < 1 || sh < 0) {   // decode needs a private tail block holding the query
             latch_error(err, kDevBounds);
             n = 1;
-            sh = 0;
         }
-        P[r] = n;   // the count for now; this thread alone touches P[r0..r1)
-        run += n;
-        mx = max(mx, n);
+        P[r] = n;
+        if (Ls) Ls[r] = L;
+    }
+    __syncthreads();
+    // exclusive prefix sum over contiguous ranges of requests per thread
+    const int per_thread = (R + kThreads - 1) / kThreads;
+    const int r0 = min(R, tid * per_thread), r1 = min(R, r0 + per_thread);
+    int32_t run = 0, mx = 0;
+    for (int r = r0; r < r1; ++r) {
+        run += P[r];
+        mx = max(mx, P[r]);
     }
     int32_t incl = run;
 #pragma unroll
@@ -239,7 +246,12 @@ __device__ void build_plan(int32_t *P, int32_t R, const int32_t *__restrict__ co
 }
 
 // The split pass: per warp, a contiguous range of the block stream through a
-// TMA ring (see the file comment).
+// TMA ring (see the file comment).  Ranges are equal in cost: a block costs
+// one unit and each segment kPieceCost more (its Q rows, its partial and the
+// ramp of a new piece), so warps whose range crosses many short segments
+// take fewer blocks.
+constexpr int32_t kPieceCost = 1;
+
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     decode_split_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
@@ -255,11 +267,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                 ~uintptr_t(1023));
     // K/V stages [kWarps][S] | Q areas [kWarps][S] | descriptors [kWarps][S] |
-    // full barriers [kWarps][S] | plan [R + 1]
+    // full barriers [kWarps][S] | plan [R + 1] | context lengths [R] (if they fit)
     const uint32_t qbase = smem_u32(smem) + (uint32_t)(kWarps * S) * kSlotBytes;
     SlotDesc *descs = reinterpret_cast<SlotDesc *>(smem + (size_t)kWarps * S * (kSlotBytes + kQBytes));
     uint64_t *bars = reinterpret_cast<uint64_t *>(descs + kWarps * S);
     int32_t *P = reinterpret_cast<int32_t *>(bars + kWarps * S);
+    int32_t *Ls = lay.lens_in_smem ? P + lay.R + 1 : nullptr;
     __shared__ int32_t s_max_n;
     __shared__ int abort_flag;
 
@@ -276,9 +289,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         fence_barrier_init();
     }
     const int32_t R = lay.R, Hkv = lay.Hkv, Hq = lay.Hq, g = lay.g;
-    build_plan(P, R, a.context_lens, a.group_of_req, a.group_blocks, a.num_groups, a.max_blocks,
+    build_plan(P, Ls, R, a.context_lens, a.group_of_req, a.group_blocks, a.num_groups, a.max_blocks,
                &s_max_n, a.err);   // ends with __syncthreads: the barriers are initialised
-    const int64_t W = (int64_t)Hkv * P[R];
+    // cost stream: segment (r, h) spans [Hkv (P[r] + c r) + h (n_r + c), + n_r + c),
+    // its blocks the last n_r positions
+    constexpr int32_t c = kPieceCost;
+    const int64_t W = (int64_t)Hkv * ((int64_t)P[R] + (int64_t)c * R);
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
     int64_t per = (W + nwarps - 1) / nwarps;
     const int64_t need = (s_max_n - 1 + kMaxPrivateParts - 3) / (kMaxPrivateParts - 2);
@@ -286,9 +302,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (per < kMinBlocksPerPiece) per = kMinBlocksPerPiece;
     const int64_t gw = (int64_t)blockIdx.x * kWarps + warp;
     const int64_t x0 = gw * per, x1 = min(x0 + per, W);
-    const int64_t nu = x1 - x0;   // units (blocks of one kv head) of this warp
 
-    if (nu > 0) {
+    if (x0 < x1) {
         float *o_part = reinterpret_cast<float *>(static_cast<char *>(a.ws) + lay.off_o);
         float2 *ml_part = reinterpret_cast<float2 *>(static_cast<char *>(a.ws) + lay.off_ml);
         int32_t *nparts = reinterpret_cast<int32_t *>(static_cast<char *>(a.ws) + lay.off_nparts);
@@ -306,10 +321,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             int lo = 0, hi = R - 1;
             while (lo < hi) {
                 const int mid = (lo + hi + 1) >> 1;
-                if (P[mid] <= xr) lo = mid; else hi = mid - 1;
+                if ((int64_t)P[mid] + (int64_t)c * mid <= xr) lo = mid; else hi = mid - 1;
             }
             const int32_t n0 = P[lo + 1] - P[lo];
-            seg_base = (int64_t)lo * Hkv + (x0 - (int64_t)Hkv * P[lo]) / n0;
+            seg_base = (int64_t)lo * Hkv + (x0 - (int64_t)Hkv * ((int64_t)P[lo] + (int64_t)c * lo)) / (n0 + c);
         }
         int32_t pr = 0, ph = 0, plo = 0, phi = 0, psh = 0, pL = 0, pn = 0, ppart = 0, pnw = 0;
         auto fill_list = [&]() {
@@ -319,16 +334,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             plo = phi = 0;
             if (pr < R) {
                 pn = P[pr + 1] - P[pr];
-                const int64_t seg_off = (int64_t)Hkv * P[pr] + (int64_t)ph * pn;
-                const int64_t lo = max(x0, seg_off), hi = min(x1, seg_off + pn);
+                // cost position of the segment's block 0
+                const int64_t b0 = (int64_t)Hkv * ((int64_t)P[pr] + (int64_t)c * pr) + (int64_t)ph * (pn + c) + c;
+                const int64_t lo = max(x0, b0), hi = min(x1, b0 + pn);
                 if (lo < hi) {
-                    plo = (int32_t)(lo - seg_off);
-                    phi = (int32_t)(hi - seg_off);
-                    pL = __ldg(a.context_lens + pr);
+                    plo = (int32_t)(lo - b0);
+                    phi = (int32_t)(hi - b0);
+                    pL = Ls ? Ls[pr] : __ldg(a.context_lens + pr);
                     const int32_t nblk = min((pL + 15) >> 4, a.max_blocks);
                     psh = max(nblk - pn, 0);
-                    ppart = lay.prefix_parts + (int32_t)(gw - seg_off / per);
-                    const int32_t n_priv = (int32_t)((seg_off + pn - 1) / per - seg_off / per + 1);
+                    ppart = lay.prefix_parts + (int32_t)(gw - b0 / per);
+                    const int32_t n_priv = (int32_t)((b0 + pn - 1) / per - b0 / per + 1);
                     const int32_t n_pre = lay.prefix_parts > 0 && a.num_groups > 0
                                               ? min((psh + lay.prefix_blocks_per_part - 1) / lay.prefix_blocks_per_part,
                                                     lay.prefix_parts)
@@ -356,7 +372,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         int k = -1, b = 0, b_lo = 0, b_hi = 0, cr = 0, ch = 0, csh = 0, cL = 0, cn = 0, cpart = 0, cnw = 0;
         int win_base = 0, nwin_for = -1;
         int32_t win = 0, nwin = 0;
-        auto enter_next = [&]() {
+        // the next piece of the range; false when the range is done
+        auto enter_next = [&]() -> bool {
             ++k;
             if (k == 32) {
                 seg_base += 32;
@@ -364,10 +381,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 k = 0;
                 nwin_for = -1;
             }
-            cr = __shfl_sync(0xffffffffu, pr, k);
-            ch = __shfl_sync(0xffffffffu, ph, k);
             b_lo = __shfl_sync(0xffffffffu, plo, k);
             b_hi = __shfl_sync(0xffffffffu, phi, k);
+            if (b_lo >= b_hi) return false;   // pieces are consecutive: none follows an empty one
+            cr = __shfl_sync(0xffffffffu, pr, k);
+            ch = __shfl_sync(0xffffffffu, ph, k);
             csh = __shfl_sync(0xffffffffu, psh, k);
             cL = __shfl_sync(0xffffffffu, pL, k);
             cn = __shfl_sync(0xffffffffu, pn, k);
@@ -386,10 +404,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     nwin_for = k + 1;
                 }
             }
+            return true;
         };
-        // issue the copies of the next block into stage s
-        auto produce = [&](int s) {
-            if (b == b_hi) enter_next();
+        // issue the copies of the next block into stage s; false when the
+        // range is done (nothing issued)
+        bool more = true;
+        auto produce = [&](int s) -> bool {
+            if (b == b_hi && !enter_next()) return false;
             if (b - win_base >= 32) {
                 win_base = b;
                 win = load_ids(cr, csh, b, b_hi);
@@ -421,25 +442,29 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             __syncwarp();
             ++b;
+            return true;
         };
 
         if (lane == 0) {
             prefetch_tmap(&tmk);
             prefetch_tmap(&tmv);
         }
-        const int64_t n_first = nu < S ? nu : (int64_t)S;
-        for (int s = 0; s < n_first; ++s) produce(s);
+        int64_t issued = 0;
+        for (int s0 = 0; s0 < S && more; ++s0) {
+            more = produce(s0);
+            if (more) ++issued;
+        }
 
         uint32_t qf[D / 16][2];
         uint4 kvn = make_uint4(0, 0, 0, 0);   // lane < CPR: k_new chunk; < 2 CPR: v_new chunk
         auto load_new = [&](const SlotDesc &d) {
             if (lane < 2 * CPR) {
                 const uint16_t *src = static_cast<const uint16_t *>(lane < CPR ? a.k_new : a.v_new);
-                const int c = lane < CPR ? lane : lane - CPR;
-                kvn = ldg16(src + ((int64_t)d.r * Hkv + d.h) * D + c * 8);
+                const int cc = lane < CPR ? lane : lane - CPR;
+                kvn = ldg16(src + ((int64_t)d.r * Hkv + d.h) * D + cc * 8);
             }
         };
-        {
+        if (issued > 0) {
             const SlotDesc d0 = mydesc[0];
             if (d0.info & kWriteSoon) load_new(d0);
         }
@@ -447,7 +472,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         int s = 0;
         uint32_t phase = 0;
         int64_t u = 0;
-        for (; u < nu; ++u) {
+        for (; u < issued; ++u) {
             if (!__all_sync(0xffffffffu, mbar_wait(mybar + 8 * s, phase, &abort_flag, kWaitLimitNs))) break;
             const SlotDesc d = mydesc[s];
             const int valid = d.info & kValidMask;
@@ -466,10 +491,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int off = valid - 1;
                 if (lane < 2 * CPR) {
                     const bool isv = lane >= CPR;
-                    const int c = isv ? lane - CPR : lane;
+                    const int cc = isv ? lane - CPR : lane;
                     uint16_t *cache = static_cast<uint16_t *>(const_cast<void *>(isv ? a.v_cache : a.k_cache));
-                    *reinterpret_cast<uint4 *>(cache + (((int64_t)d.phys * Hkv + d.h) * 16 + off) * D + c * 8) = kvn;
-                    const uint32_t dst = (isv ? vb : kb) + tile_off(off, c);
+                    *reinterpret_cast<uint4 *>(cache + (((int64_t)d.phys * Hkv + d.h) * 16 + off) * D + cc * 8) = kvn;
+                    const uint32_t dst = (isv ? vb : kb) + tile_off(off, cc);
                     asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(dst), "r"(kvn.x), "r"(kvn.y),
                                  "r"(kvn.z), "r"(kvn.w)
                                  : "memory");
@@ -479,12 +504,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // keys past the context: p = 0, but their V rows may hold
                 // anything (0 * NaN = NaN in the MMA), so clear them
                 for (int i = lane; i < (16 - max(valid, 0)) * CPR; i += 32) {
-                    const int row = max(valid, 0) + i / CPR, c = i % CPR;
-                    asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};" ::"r"(vb + tile_off(row, c)), "r"(0)
+                    const int row = max(valid, 0) + i / CPR, cc = i % CPR;
+                    asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};" ::"r"(vb + tile_off(row, cc)), "r"(0)
                                  : "memory");
                 }
             }
-            if (u + 1 < nu) {
+            if (u + 1 < issued) {
                 // a piece that starts next and ends with the query token's
                 // row: its new K/V in flight from now on
                 const SlotDesc d1 = mydesc[s + 1 == S ? 0 : s + 1];
@@ -502,34 +527,37 @@ __global__ void __launch_bounds__(kThreads, 1)
                     l1 += __shfl_xor_sync(0xffffffffu, l1, off);
                 }
 #pragma unroll
-                for (int c = 0; c < 2; ++c) {
-                    const int hd = 2 * (lane & 3) + c;
+                for (int cc = 0; cc < 2; ++cc) {
+                    const int hd = 2 * (lane & 3) + cc;
                     if (hd < g) {
                         const int64_t slot = ((int64_t)d.r * Hq + d.h * g + hd) * lay.parts_per_head + d.part;
                         float *dst = o_part + slot * D + (lane >> 2);
 #pragma unroll
                         for (int mt = 0; mt < D / 16; ++mt) {
-                            dst[16 * mt] = st.o[mt][c];
-                            dst[16 * mt + 8] = st.o[mt][2 + c];
+                            dst[16 * mt] = st.o[mt][cc];
+                            dst[16 * mt + 8] = st.o[mt][2 + cc];
                         }
-                        if ((lane >> 2) == 0) ml_part[slot] = make_float2(st.m[c], c ? l1 : l0);
+                        if ((lane >> 2) == 0) ml_part[slot] = make_float2(st.m[cc], cc ? l1 : l0);
                     }
                 }
             }
             __syncwarp();
-            if (u + S < nu) produce(s);
+            if (more) {
+                more = produce(s);
+                if (more) ++issued;
+            }
             if (++s == S) {
                 s = 0;
                 phase ^= 1u;
             }
         }
-        if (u < nu) {
+        if (u < issued) {
             // a wait ran out: latch it, then let this warp's copies still in
-            // flight (units u .. u + S - 1) land before the CTA exits
+            // flight (units u .. issued - 1) land before the CTA exits
             if (lane == 0) {
                 latch_error(a.err, kDevTimeout);
                 int quiet = 0;
-                for (int64_t v = u; v < nu && v < u + S; ++v) {
+                for (int64_t v = u; v < issued; ++v) {
                     const int sv = (int)(v % S);
                     mbar_wait(mybar + 8 * sv, (uint32_t)((v / S) & 1), &quiet, kDrainLimitNs);
                 }
@@ -652,9 +680,10 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(DecodeArgs a, Decod
 namespace {
 
 // Shared memory of the split pass for `stages` ring stages.
-size_t split_smem_bytes(int32_t R, int32_t d, int stages) {
+size_t split_smem_bytes(int32_t R, int32_t d, int stages, bool lens) {
     const size_t slot = 2 * (size_t)(d / 64) * 2048 + 8 * (size_t)d * 2;   // K/V tiles + Q area
-    return 1024 + (size_t)kWarps * stages * (slot + sizeof(SlotDesc) + 8) + 4 * ((size_t)R + 1);
+    return 1024 + (size_t)kWarps * stages * (slot + sizeof(SlotDesc) + 8) + 4 * ((size_t)R + 1) +
+           (lens ? 4 * (size_t)R : 0);
 }
 
 }  // namespace
@@ -671,22 +700,26 @@ DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_
     L.prefix_ctas = 0;
     L.prefix_early = 0;
     // the private split pass streams about kSplitGBsPerSM per SM, together
-    // at most kSplitGBsTotal; its bytes are estimated from the table width
-    // (60 % of the blocks past the longest prefix), which only steers choices
-    constexpr double kSplitGBsPerSM = 50.0, kSplitGBsTotal = 6600.0;
+    // at most kSplitGBsTotal, after about kSplitStartUs of start-up; its bytes
+    // are estimated from the table width (60 % of the blocks past the longest
+    // prefix), which only steers choices
+    constexpr double kSplitGBsPerSM = 47.0, kSplitGBsTotal = 6300.0, kSplitStartUs = 7.0;
     const double unit_bytes = 16.0 * d * 2 * 2;   // K + V of one (block, kv head)
     const double priv_blocks = 0.6 * std::max(1, max_blocks - std::max(0, max_group_blocks));
     const double split_bytes = (double)R * Hkv * priv_blocks * unit_bytes;
-    auto split_us = [&](int nsm) { return split_bytes / std::min(kSplitGBsTotal, kSplitGBsPerSM * nsm) * 1e-3; };
+    auto split_us = [&](int nsm) {
+        return kSplitStartUs + split_bytes / std::min(kSplitGBsTotal, kSplitGBsPerSM * nsm) * 1e-3;
+    };
     if (num_groups > 0 && max_group_blocks > 0 && max_group_members > 0) {
         // Key splits of the prefix pass: one CTA per (group, kv head, member
         // tile, split), one CTA per SM.  When its grid leaves at least a
         // quarter of the SMs free, the split pass runs beside it on those
         // SMs and a step costs about max(prefix critical path, split time on
         // the free SMs); otherwise the two run one after the other.
-        // Measured on GB300: a prefix CTA costs about 16 us of fixed work
-        // (set-up, Q tile, pipeline fill, partial writes, with the split pass
-        // loading HBM beside it) plus 2.1 us per key tile.
+        // Measured on GB300 with per-CTA clock stamps: a prefix CTA costs about
+        // 16 us of fixed work (set-up, Q tile, pipeline fill, partial writes)
+        // plus 1.8 us per key tile alone, 3.1 us with the split pass loading
+        // HBM beside it (its 2-stage K/V ring then waits on memory).
         const int per_item = 2 * (128 / L.g);   // members per work item (two 128-row tiles)
         const int64_t tiles = (int64_t)num_groups * Hkv * ((max_group_members + per_item - 1) / per_item);
         const int key_tiles = (max_group_blocks + 7) / 8;
@@ -695,10 +728,10 @@ DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_
         for (int sp = 1; sp <= kMaxPrefixParts && sp <= key_tiles; ++sp) {
             const int per = (key_tiles + sp - 1) / sp;
             const int64_t ctas = tiles * sp;
-            const double cta_us = 16.0 + 2.1 * per;
+            const bool beside = 4 * ctas <= 3 * (int64_t)sms;
+            const double cta_us = 16.0 + (beside ? 3.1 : 1.8) * per;
             const double crit = (double)((ctas + sms - 1) / sms) * cta_us;
-            const double t = (4 * ctas <= 3 * (int64_t)sms) ? std::max(crit, split_us(sms - (int)ctas))
-                                                           : crit + split_us(sms);
+            const double t = beside ? std::max(crit, split_us(sms - (int)ctas)) : crit + split_us(sms);
             if (t < best_t - 1e-9) { best_t = t; best = sp; }
         }
         const int per_tiles = (key_tiles + best - 1) / best;
@@ -712,8 +745,10 @@ DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_
     L.stages = 2;
     const int max_stages = d == 64 ? 4 : 3;
     for (int st = max_stages; st > 2; --st)
-        if (split_smem_bytes(R, d, st) <= kMaxSmemPerBlock) { L.stages = st; break; }
-    L.split_smem = split_smem_bytes(R, d, L.stages);
+        if (split_smem_bytes(R, d, st, false) <= kMaxSmemPerBlock) { L.stages = st; break; }
+    // the context lengths beside the plan when they fit (saves a global read per piece list)
+    L.lens_in_smem = split_smem_bytes(R, d, L.stages, true) <= kMaxSmemPerBlock ? 1 : 0;
+    L.split_smem = split_smem_bytes(R, d, L.stages, L.lens_in_smem != 0);
     L.parts_per_head = L.prefix_parts + kMaxPrivateParts;
     const size_t slots = (size_t)R * Hq * L.parts_per_head;
     auto up = [](size_t x) { return (x + 255) & ~(size_t)255; };

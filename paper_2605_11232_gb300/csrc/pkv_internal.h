@@ -107,6 +107,7 @@ struct DecodeLayout {
     int32_t prefix_early;        // the prefix pass lets the split pass start beside it
     int32_t split_grid;          // split-pass CTAs beside an early prefix pass
     int32_t stages;              // ring stages per warp of the split pass
+    int32_t lens_in_smem;        // the split pass keeps the context lengths in shared memory
     size_t split_smem;           // dynamic shared memory of the split pass
     int32_t parts_per_head;      // prefix_parts + kMaxPrivateParts
     // byte offsets inside the workspace
