@@ -339,17 +339,15 @@ def measure_workload(name, steps, warmup, use_groups=True, e2e_steps=0):
 
     if e2e_steps and Rd and not Rp:
         # End to end through the C ABI from host buffers, as a serving loop
-        # runs it: every step computes the slot mapping on the host (into the
-        # pinned step buffer), then one paged_attn_decode_step call copies the
-        # step's packed inputs (q, new K/V, slots, context lengths) to the
-        # device, writes the new tokens, decodes and copies the output back to
-        # pinned memory.  Alternate steps go to two streams, each with its own
+        # runs it: one paged_attn_decode_step call per step copies the step's
+        # packed inputs (q, new K/V, context lengths) to the device, decodes
+        # with the new tokens stored by the decode kernels
+        # (PKV_STEP_FUSED_WRITE) and copies the output back to pinned memory.  Alternate steps go to two streams, each with its own
         # device input and output buffers; a step's kernels wait for the
         # previous step's (one decode per pool at a time), so its copies
         # overlap the other stream's kernels.  A pinned buffer is refilled
         # only after the step that last used it has completed.
-        layout, host, _ = B.step_buffers(b, copies=2)
-        slot_np = [B.step_view(h, layout.slot_mapping, b.slots).numpy() for h in host]
+        layout, host, _ = B.step_buffers(b, copies=2, fused=True)
         dev = [torch.empty(layout.bytes, dtype=torch.uint8, device=b.device) for _ in range(2)]
         for k in range(2):
             dev[k].copy_(host[k])
@@ -371,7 +369,6 @@ def measure_workload(name, steps, warmup, use_groups=True, e2e_steps=0):
             k = i & 1
             if events[k] is not None:
                 events[k].synchronize()   # the step that last used buffer k is done
-            pkv.kv_slot_mapping(b.pool, b.table_host, w.context_lens, w.new_lens, out=slot_np[k])
             steps_k[k]()
             ev = torch.cuda.Event()
             ev.record(streams[k])
@@ -392,6 +389,130 @@ def measure_workload(name, steps, warmup, use_groups=True, e2e_steps=0):
     del b, flush_buf, ws
     torch.cuda.empty_cache()
     return res
+
+
+def _timed(step, flush, steps, warmup, stream):
+    import torch
+    for _ in range(warmup):
+        flush()
+        step()
+    torch.cuda.synchronize()
+    return run_steps(step, flush, steps, stream)
+
+
+def measure_verify(steps, warmup, k=8):
+    """Speculative verification of tree-shaped drafts (Sec. 5.3) on the
+    Llama-3-8B-shaped decode batch: every request carries k draft tokens in a
+    seeded tree (chains, stars and random trees in turn) over its cached
+    context (64 requests, shared 4096-token prefix).  A step writes the drafts'
+    K/V (kv_cache_write) and runs paged_attn_verify_tree.  Reported: TFLOP/s on
+    visible (query, key) pairs, and GB/s on distinct K/V bytes (shared prefix
+    once) + Q/O + the write."""
+    import numpy as np
+    import torch
+
+    from paper_2605_11232_gb300 import batch as B
+    from paper_2605_11232_gb300 import pkv
+    from paper_2605_11232_gb300.workloads import make_workload
+
+    w0 = make_workload("l8b_decode", values=False)
+    R = w0.num_requests
+    cached = [int(c) for c in w0.cached_lens]
+    w = make_workload("custom", seed=31, custom=dict(
+        Hq=w0.num_q_heads, Hkv=w0.num_kv_heads, d=w0.head_dim, prefix_lens=list(w0.prefix_lens),
+        group=[int(x) for x in w0.group_of_req], cached=cached, new=[k] * R, decode=[False] * R))
+    rng = np.random.default_rng(31)
+    parents = []
+    for r in range(R):
+        if r % 3 == 0:
+            parents += [-1] + list(range(k - 1))
+        elif r % 3 == 1:
+            parents += [-1] * k
+        else:
+            parents += [int(rng.integers(-1, i)) if i else -1 for i in range(k)]
+    cu = np.arange(0, R * k + 1, k, dtype=np.int32)
+    masks_np = pkv.pkv_tree_masks(np.asarray(parents, np.int32), cu)
+    b = B.build_batch(w, poison=False)
+    masks = torch.from_numpy(masks_np).to(b.device)
+    T = R * k
+    out = torch.empty((T, w.num_q_heads, w.head_dim), dtype=torch.bfloat16, device=b.device)
+    flush_buf = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=b.device)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        B.run_write(b)
+        pkv.paged_attn_verify_tree(b.pool, b.q, out, None, b.cu_pre, b.context_lens, b.table, k, w.scale, masks)
+
+    ms = _timed(step, lambda: flush_buf.fill_(1), steps, warmup, stream)
+    pkv.pkv_trace_enable(b.pool, True)
+    _timed(step, lambda: flush_buf.fill_(1), 2, 1, stream)
+    pkv.pkv_trace_read(b.pool)
+    run_steps(step, lambda: flush_buf.fill_(1), steps, stream)
+    trace = pkv.pkv_trace_read(b.pool)
+    pkv.pkv_trace_enable(b.pool, False)
+    assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
+    # visible pairs: each draft sees its cached context and its ancestors (itself included)
+    pairs = 0
+    for r in range(R):
+        for i in range(k):
+            pairs += cached[r] + bin(int(masks_np[r * k + i])).count("1")
+    flops = 4 * w.head_dim * w.num_q_heads * pairs
+    kv_rows = sum(w.prefix_lens) + sum(c - w.prefix_len_of(r) for r, c in enumerate(cached)) + T
+    nbytes = kv_rows * kv_row_bytes(w) + 2 * T * w.num_q_heads * w.head_dim * 2 + write_bytes(w, T)
+    n_v, t_v = trace["prefill"]
+    v_ms = t_v / n_v
+    b.close()
+    mean = statistics.mean(ms)
+    return {"ms_per_step": mean, "drafts_per_request": k, "requests": R,
+            "verify_kernel_us": v_ms * 1e3, "verify_tflops": flops / (v_ms * 1e-3) / 1e12,
+            "step_hbm_gbs": nbytes / (mean * 1e-3) / 1e9,
+            "kernels": {kk: {"launches": n, "avg_us": 1e3 * t / n} for kk, (n, t) in trace.items()},
+            "note": "trees: chains, stars and seeded random trees in turn; drafts' K/V written by "
+                    "kv_cache_write in the step"}
+
+
+def measure_transfer(steps, warmup):
+    """KV-block transfer (prefill/decode disaggregation, Sec. 2 / Sec. 7): the
+    Llama-3-8B-shaped suffix-prefill batch's blocks (32 requests, shared 4096
+    prefix once) gathered from its pool into a staging buffer and scattered
+    into another pool's blocks, one GPU.  GB/s on 2 x (read + write) bytes
+    of every moved block."""
+    import numpy as np
+    import torch
+
+    from paper_2605_11232_gb300 import batch as B
+    from paper_2605_11232_gb300 import pkv
+    from paper_2605_11232_gb300.workloads import make_workload
+
+    w = make_workload("l8b_prefill")
+    b = B.build_batch(w, poison=False)
+    B.run_write(b)
+    ids = np.unique(np.concatenate([b.table_host[r, :(int(w.context_lens[r]) + 15) // 16]
+                                    for r in range(w.num_requests)])).astype(np.int32)
+    n = len(ids)
+    dk = torch.empty((n,) + tuple(b.k_cache.shape[1:]), dtype=torch.bfloat16, device=b.device)
+    dv = torch.empty_like(dk)
+    dst = pkv.kv_pool_create(n, w.num_kv_heads, w.head_dim, dk, dv, placement_seed=5)
+    dst_ids = torch.from_numpy(pkv.kv_pool_alloc(dst, n)).to(b.device)
+    src_ids = torch.from_numpy(ids).to(b.device)
+    staging = torch.empty(pkv.pkv_blocks_staging_size(b.pool, n), dtype=torch.uint8, device=b.device)
+    flush_buf = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=b.device)
+
+    def step():
+        pkv.pkv_blocks_gather(b.pool, src_ids, staging)
+        pkv.pkv_blocks_scatter(dst, dst_ids, staging)
+
+    ms = _timed(step, lambda: flush_buf.fill_(1), steps, warmup, torch.cuda.current_stream())
+    assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK and pkv.pkv_check_device_errors(dst) == pkv.PKV_OK
+    assert torch.equal(dk[dst_ids.long()].view(torch.int16), b.k_cache[src_ids.long()].view(torch.int16))
+    moved = staging.numel()            # bytes of the moved blocks
+    mean = statistics.mean(ms)
+    pkv.kv_pool_destroy(dst)
+    b.close()
+    return {"ms_per_step": mean, "blocks": n, "bytes_moved": moved,
+            "transfer_hbm_gbs": 4 * moved / (mean * 1e-3) / 1e9,
+            "note": "one GPU: source and destination pools on the same device (the cross-GPU copy "
+                    "of the staging buffer is not measured)"}
 
 
 def summarize(res, peaks):
@@ -551,6 +672,17 @@ def main():
             try:
                 r = measure_workload(name, max(10, args.steps // 10), 3)
                 extra[name] = summarize(r, peaks)
+            except Exception as e:   # report, do not hide
+                extra[name] = {"error": str(e)}
+        for name, fn in (("spec_verify_tree", measure_verify), ("pd_block_transfer", measure_transfer)):
+            try:
+                r = fn(max(10, args.steps // 10), 3)
+                if "transfer_hbm_gbs" in r:
+                    r["frac_of_measured_hbm"] = r["transfer_hbm_gbs"] / peaks[0]
+                if "verify_tflops" in r:
+                    r["verify_frac_of_measured_bf16"] = r["verify_tflops"] / peaks[1]
+                    r["step_frac_of_measured_hbm"] = r["step_hbm_gbs"] / peaks[0]
+                extra[name] = r
             except Exception as e:   # report, do not hide
                 extra[name] = {"error": str(e)}
     clocks.stop()

@@ -309,6 +309,32 @@ int paged_attn_prefill(pkv_pool_t pool, const void *q, void *out, float *lse,
                        int32_t max_seqlen_q, int32_t num_q_heads, float scale,
                        pkv_stream_t stream);
 
+/* ---- speculative-decode verification with tree-shaped drafts (device) ---- */
+
+/* paged_attn_prefill where each request's new tokens are draft tokens of a
+ * tree (Sec. 5.3: speculative decoding verifies several drafts in one pass):
+ * new token i of a request sees every context token and exactly the new
+ * tokens j whose bit j is set in tree_mask[cu_seqlens_q[r] + i] (its
+ * ancestors and itself; pkv_tree_masks builds them from parent indices).
+ * tree_mask: device uint64 [T], 8-byte aligned.  At most 64 new tokens per
+ * request (max_seqlen_q <= 64, else UNSUPPORTED).  Every other argument,
+ * layout and error as paged_attn_prefill.  A chain mask (bits 0..i for token
+ * i) gives paged_attn_prefill's causal result. */
+int paged_attn_verify_tree(pkv_pool_t pool, const void *q, void *out, float *lse,
+                           const int32_t *cu_seqlens_q, const int32_t *context_lens,
+                           const int32_t *block_table, int32_t max_blocks, int32_t num_requests,
+                           int32_t max_seqlen_q, int32_t num_q_heads, float scale,
+                           const uint64_t *tree_mask, pkv_stream_t stream);
+
+/* Draft masks of tree-shaped drafts (host): parent[cu_seqlens[r] + i] is the
+ * draft that draft i of request r continues (-1: the context), an earlier
+ * draft of the same request; masks_out[cu_seqlens[r] + i] gets bit j set for
+ * each draft j on i's path, itself included.  parent, cu_seqlens
+ * ([num_requests + 1], cu_seqlens[0] = 0), masks_out: host arrays.  At most
+ * 64 drafts per request.  Errors: INVALID_ARG. */
+int pkv_tree_masks(const int32_t *parent, const int32_t *cu_seqlens, int32_t num_requests,
+                   uint64_t *masks_out);
+
 /* ---- a5-a7: decode (device) ---------------------------------------------- */
 
 /* Bytes of workspace paged_attn_decode needs for these shapes (host call).
@@ -367,7 +393,14 @@ int paged_attn_decode_append(pkv_pool_t pool, const void *q, const void *k_new, 
 typedef struct pkv_step_layout {
     size_t q, k_new, v_new, slot_mapping, context_lens;
     size_t bytes;
+    uint64_t flags;   /* PKV_STEP_* */
 } pkv_step_layout;
+
+/* The step's new tokens are the requests' query tokens (num_new_tokens ==
+ * num_requests, token r at position context_lens[r] - 1): the decode kernels
+ * store them (paged_attn_decode_append) instead of kv_cache_write; the
+ * slot_mapping region is not read. */
+#define PKV_STEP_FUSED_WRITE 1u
 
 /* One decode step of a serving loop from host memory (Sec. 5.3's decode with
  * the paged cache of Sec. 5.4), all enqueued on `stream`; the call does not
@@ -375,7 +408,8 @@ typedef struct pkv_step_layout {
  *   1. one copy of layout->bytes bytes from host_in to dev_in (host_in should
  *      be pinned for the copy to be asynchronous; dev_in is device memory,
  *      16-byte aligned, with the same layout),
- *   2. kv_cache_write of the T = num_new_tokens new tokens in dev_in,
+ *   2. kv_cache_write of the T = num_new_tokens new tokens in dev_in (with
+ *      PKV_STEP_FUSED_WRITE in layout->flags: stored by step 3 instead),
  *   3. paged_attn_decode of the R = num_requests queries in dev_in over
  *      block_table (device int32 [R][max_blocks]) into out (device bf16) and
  *      lse (device fp32, or NULL),
@@ -460,6 +494,38 @@ int pkv_trace_enable(pkv_pool_t pool, int32_t enable);
 int pkv_trace_read(pkv_pool_t pool, pkv_kernel_time *out, int32_t max_entries, int32_t *n_out);
 
 /* ---- errors --------------------------------------------------------------- */
+
+/* ---- KV-block transfer between pools (device) -------------------------------- */
+
+/* Prefill/decode disaggregation (Sec. 2; Sec. 7) moves a request's KV blocks
+ * from the pool of the instance that prefilled it to the pool of the one that
+ * decodes it.  The blocks are gathered into one contiguous staging buffer
+ * (the unit a peer or network copy moves) and scattered from it into blocks
+ * allocated in the destination pool (kv_pool_alloc); the caller then
+ * releases the source blocks (kv_pool_release), which moves the references.
+ * Staging layout: [n][2][num_kv_heads][16][head_dim] bf16, block i's K tile
+ * (all kv heads) then its V tile: the blocks' bytes as they are in the
+ * pools, so both copies are bit-exact.  The two pools need the same
+ * num_kv_heads and head_dim.  The paper gives the mechanism, not a layout or
+ * an interface; these calls are this library's.
+ *
+ * Bytes of staging for n blocks of this pool's geometry (host call). */
+int pkv_blocks_staging_size(pkv_pool_t pool, int32_t n, size_t *bytes_out);
+
+/* Copy the n blocks block_ids[0..n) of the pool into staging.
+ *  block_ids: device int32 [n]; an id outside [0, num_blocks) is skipped and
+ *  latches DEVICE_BOUNDS.
+ *  staging: device, 16-byte aligned, pkv_blocks_staging_size(n) bytes.
+ * Asynchronous on `stream`.  Errors: INVALID_ARG, CUDA. */
+int pkv_blocks_gather(pkv_pool_t pool, const int32_t *block_ids, int32_t n, void *staging,
+                      pkv_stream_t stream);
+
+/* Copy staging (as written by pkv_blocks_gather) into the n blocks
+ * block_ids[0..n) of the pool: every K and V row of each block.  The target
+ * blocks should be allocated and private (reference count 1): shared blocks
+ * are immutable.  Arguments, bounds and errors as pkv_blocks_gather. */
+int pkv_blocks_scatter(pkv_pool_t pool, const int32_t *block_ids, int32_t n, const void *staging,
+                       pkv_stream_t stream);
 
 /* Synchronise `stream`, then read and clear the pool's device error word.
  * *code_out gets PKV_OK or the first latched device status (DEVICE_BOUNDS,

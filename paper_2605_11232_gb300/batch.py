@@ -178,19 +178,20 @@ def step_view(buf: torch.Tensor, off: int, like: torch.Tensor) -> torch.Tensor:
     return buf[off:off + nb].view(like.dtype).view(like.shape)
 
 
-def step_buffers(b: Batch, copies: int = 2):
+def step_buffers(b: Batch, copies: int = 2, fused: bool = False):
     """Packed inputs of one decode step of a decode-only batch (q, new K/V,
     slot mapping, context lengths; 256-byte aligned regions): the
     pkv.StepLayout, `copies` pinned host buffers holding them, and a device
-    buffer of the same size."""
+    buffer of the same size.  fused: the decode kernels store the new K/V
+    (PKV_STEP_FUSED_WRITE), and the packed buffer holds no slot mapping."""
     if b.pre.stop != b.pre.start:
         raise ValueError("step buffers are for decode-only batches")
-    parts = step_parts(b)
+    parts = [pt for pt in step_parts(b) if not (fused and pt[0] == "slot_mapping")]
     offs, n = {}, 0
     for name, t in parts:
         offs[name] = n
         n += (t.numel() * t.element_size() + 255) // 256 * 256
-    layout = pkv.StepLayout(bytes=n, **offs)
+    layout = pkv.StepLayout(bytes=n, flags=pkv.PKV_STEP_FUSED_WRITE if fused else 0, **offs)
     hosts = [torch.empty(n, dtype=torch.uint8).pin_memory() for _ in range(copies)]
     for h in hosts:
         for name, t in parts:

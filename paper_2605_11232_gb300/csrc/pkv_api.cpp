@@ -19,7 +19,7 @@
 
 namespace pkv {
 const char *const kKernelNames[kNumKernelIds] = {"kv_cache_write", "decode_split", "decode_combine",
-                                                 "decode_prefix", "prefill"};
+                                                 "decode_prefix", "prefill", "block_copy"};
 }
 
 namespace {
@@ -428,11 +428,15 @@ int kv_cache_write(pkv_pool_t pool, const void *k_new, const void *v_new,
     return ok();
 }
 
-int paged_attn_prefill(pkv_pool_t pool, const void *q, void *out, float *lse,
-                       const int32_t *cu_seqlens_q, const int32_t *context_lens,
-                       const int32_t *block_table, int32_t max_blocks, int32_t num_requests,
-                       int32_t max_seqlen_q, int32_t num_q_heads, float scale,
-                       pkv_stream_t stream) {
+}  // extern "C"
+
+namespace {
+
+// paged_attn_prefill, with tree-shaped draft masks when tree_mask is set
+int prefill_impl(pkv_pool_t pool, const void *q, void *out, float *lse, const int32_t *cu_seqlens_q,
+                 const int32_t *context_lens, const int32_t *block_table, int32_t max_blocks,
+                 int32_t num_requests, int32_t max_seqlen_q, int32_t num_q_heads, float scale,
+                 const uint64_t *tree_mask, pkv_stream_t stream) {
     int rc = check_kernel_pool(pool);
     if (rc != PKV_OK) return rc;
     const pkv_pool_desc &d = pool->desc;
@@ -462,8 +466,56 @@ int paged_attn_prefill(pkv_pool_t pool, const void *q, void *out, float *lse,
     a.scale_log2 = scale * 1.4426950408889634f;
     a.tmap_k = &pool->tmap_k; a.tmap_v = &pool->tmap_v;
     a.err = pool->d_err;
+    a.tree_mask = reinterpret_cast<const unsigned long long *>(tree_mask);
     cudaError_t e = pkv::launch_prefill(a, static_cast<cudaStream_t>(stream), pool->tracer);
     if (e != cudaSuccess) return cuda_fail(e, "paged_attn_prefill launch");
+    return ok();
+}
+
+}  // namespace
+
+extern "C" {
+
+int paged_attn_prefill(pkv_pool_t pool, const void *q, void *out, float *lse,
+                       const int32_t *cu_seqlens_q, const int32_t *context_lens,
+                       const int32_t *block_table, int32_t max_blocks, int32_t num_requests,
+                       int32_t max_seqlen_q, int32_t num_q_heads, float scale,
+                       pkv_stream_t stream) {
+    return prefill_impl(pool, q, out, lse, cu_seqlens_q, context_lens, block_table, max_blocks,
+                        num_requests, max_seqlen_q, num_q_heads, scale, nullptr, stream);
+}
+
+int paged_attn_verify_tree(pkv_pool_t pool, const void *q, void *out, float *lse,
+                           const int32_t *cu_seqlens_q, const int32_t *context_lens,
+                           const int32_t *block_table, int32_t max_blocks, int32_t num_requests,
+                           int32_t max_seqlen_q, int32_t num_q_heads, float scale,
+                           const uint64_t *tree_mask, pkv_stream_t stream) {
+    if (max_seqlen_q > 64) return fail(PKV_ERR_UNSUPPORTED, "at most 64 draft tokens per request");
+    if (num_requests > 0 && max_seqlen_q > 0 &&
+        (!tree_mask || (reinterpret_cast<uintptr_t>(tree_mask) & 7)))
+        return fail(PKV_ERR_INVALID_ARG, "tree_mask must be a non-NULL, 8-byte aligned device array");
+    return prefill_impl(pool, q, out, lse, cu_seqlens_q, context_lens, block_table, max_blocks,
+                        num_requests, max_seqlen_q, num_q_heads, scale, tree_mask, stream);
+}
+
+int pkv_tree_masks(const int32_t *parent, const int32_t *cu_seqlens, int32_t num_requests,
+                   uint64_t *masks_out) {
+    if (num_requests < 0 || !cu_seqlens || (num_requests > 0 && cu_seqlens[num_requests] > 0 &&
+                                             (!parent || !masks_out)))
+        return fail(PKV_ERR_INVALID_ARG, "bad arguments");
+    if (cu_seqlens[0] != 0) return fail(PKV_ERR_INVALID_ARG, "cu_seqlens[0] must be 0");
+    for (int32_t r = 0; r < num_requests; ++r) {
+        const int32_t a = cu_seqlens[r], n = cu_seqlens[r + 1] - a;
+        if (n < 0 || n > 64)
+            return fail(PKV_ERR_INVALID_ARG, "request %d: %d drafts (0 to 64 allowed)", r, n);
+        for (int32_t i = 0; i < n; ++i) {
+            const int32_t pa = parent[a + i];
+            if (pa < -1 || pa >= i)
+                return fail(PKV_ERR_INVALID_ARG, "request %d draft %d: parent %d is not -1 or an earlier draft",
+                            r, i, pa);
+            masks_out[a + i] = (pa < 0 ? 0ull : masks_out[a + pa]) | (1ull << i);
+        }
+    }
     return ok();
 }
 
@@ -609,12 +661,16 @@ int paged_attn_decode_step(pkv_pool_t pool, const void *host_in, void *dev_in,
     if (!aligned16(dev_in)) return fail(PKV_ERR_INVALID_ARG, "dev_in must be 16-byte aligned");
     const pkv_pool_desc &d = pool->desc;
     const size_t row = (size_t)d.head_dim * 2;
+    const bool fused = (layout->flags & PKV_STEP_FUSED_WRITE) != 0;
+    if (layout->flags & ~(uint64_t)PKV_STEP_FUSED_WRITE) return fail(PKV_ERR_INVALID_ARG, "unknown step flags");
+    if (fused && num_new_tokens != num_requests)
+        return fail(PKV_ERR_INVALID_ARG, "a fused-write step has one new token per request");
     // every region 16-byte aligned and inside the buffer
     const struct { size_t off, len; } regions[] = {
         {layout->q, (size_t)num_requests * num_q_heads * row},
         {layout->k_new, (size_t)num_new_tokens * d.num_kv_heads * row},
         {layout->v_new, (size_t)num_new_tokens * d.num_kv_heads * row},
-        {layout->slot_mapping, (size_t)num_new_tokens * sizeof(int64_t)},
+        {fused ? 0 : layout->slot_mapping, fused ? 0 : (size_t)num_new_tokens * sizeof(int64_t)},
         {layout->context_lens, (size_t)num_requests * sizeof(int32_t)},
     };
     for (const auto &g : regions)
@@ -626,7 +682,8 @@ int paged_attn_decode_step(pkv_pool_t pool, const void *host_in, void *dev_in,
     pkv::DecodeLayout L{};
     pkv::DecodeArgs a{};
     bool empty = true;
-    rc = prepare_decode(pool, din + layout->q, nullptr, nullptr, out, lse,
+    rc = prepare_decode(pool, din + layout->q, fused ? din + layout->k_new : nullptr,
+                        fused ? din + layout->v_new : nullptr, out, lse,
                         reinterpret_cast<const int32_t *>(din + layout->context_lens), block_table,
                         max_blocks, num_requests, num_q_heads, scale, groups, workspace, workspace_bytes,
                         &L, &a, &empty);
@@ -639,10 +696,12 @@ int paged_attn_decode_step(pkv_pool_t pool, const void *host_in, void *dev_in,
         e = cudaStreamWaitEvent(st, static_cast<cudaEvent_t>(wait_event), 0);
         if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode_step wait_event");
     }
-    rc = kv_cache_write(pool, din + layout->k_new, din + layout->v_new,
-                        reinterpret_cast<const int64_t *>(din + layout->slot_mapping), num_new_tokens,
-                        stream);
-    if (rc != PKV_OK) return rc;
+    if (!fused) {
+        rc = kv_cache_write(pool, din + layout->k_new, din + layout->v_new,
+                            reinterpret_cast<const int64_t *>(din + layout->slot_mapping), num_new_tokens,
+                            stream);
+        if (rc != PKV_OK) return rc;
+    }
     if (!empty) {
         e = pkv::launch_decode(L, a, d.num_blocks, st, pool->tracer);
         if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode_step launch");
@@ -660,6 +719,51 @@ int paged_attn_decode_step(pkv_pool_t pool, const void *host_in, void *dev_in,
         if (e != cudaSuccess) return cuda_fail(e, "paged_attn_decode_step output copy");
     }
     return ok();
+}
+
+int pkv_blocks_staging_size(pkv_pool_t pool, int32_t n, size_t *bytes_out) {
+    if (!pool || n < 0 || !bytes_out) return fail(PKV_ERR_INVALID_ARG, "bad arguments");
+    *bytes_out = (size_t)n * 2 * pool->desc.num_kv_heads * 16 * pool->desc.head_dim * 2;
+    return ok();
+}
+
+}  // extern "C"
+
+namespace {
+
+int block_copy(pkv_pool_t pool, const int32_t *block_ids, int32_t n, void *staging, bool to_staging,
+               pkv_stream_t stream, const char *what) {
+    int rc = check_kernel_pool(pool);
+    if (rc != PKV_OK) return rc;
+    if (n < 0) return fail(PKV_ERR_INVALID_ARG, "%s: n < 0", what);
+    if (n == 0) return ok();
+    if (!block_ids || !staging) return fail(PKV_ERR_INVALID_ARG, "%s: NULL buffer", what);
+    if ((reinterpret_cast<uintptr_t>(block_ids) & 3) || !aligned16(staging))
+        return fail(PKV_ERR_INVALID_ARG, "%s: misaligned block ids or staging", what);
+    if ((rc = set_device(pool)) != PKV_OK) return rc;
+    const pkv_pool_desc &d = pool->desc;
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (pool->tracer) pool->tracer->begin(pkv::kKernelBlockCopy, st);
+    cudaError_t e = pkv::launch_block_copy(block_ids, n, d.num_kv_heads, d.head_dim, pool->k_cache,
+                                           pool->v_cache, staging, d.num_blocks, to_staging, pool->d_err,
+                                           pool->num_sms, st);
+    if (pool->tracer) pool->tracer->end(pkv::kKernelBlockCopy, st);
+    if (e != cudaSuccess) return cuda_fail(e, what);
+    return ok();
+}
+
+}  // namespace
+
+extern "C" {
+
+int pkv_blocks_gather(pkv_pool_t pool, const int32_t *block_ids, int32_t n, void *staging,
+                      pkv_stream_t stream) {
+    return block_copy(pool, block_ids, n, staging, true, stream, "pkv_blocks_gather");
+}
+
+int pkv_blocks_scatter(pkv_pool_t pool, const int32_t *block_ids, int32_t n, const void *staging,
+                       pkv_stream_t stream) {
+    return block_copy(pool, block_ids, n, const_cast<void *>(staging), false, stream, "pkv_blocks_scatter");
 }
 
 int pkv_check_device_errors(pkv_pool_t pool, pkv_stream_t stream, int32_t *code_out) {

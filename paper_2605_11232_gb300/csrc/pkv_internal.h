@@ -20,7 +20,8 @@ enum KernelId : int {
     kKernelDecodeCombine = 2,
     kKernelDecodePrefix = 3,
     kKernelPrefill = 4,
-    kNumKernelIds = 5,
+    kKernelBlockCopy = 5,
+    kNumKernelIds = 6,
 };
 extern const char *const kKernelNames[kNumKernelIds];
 
@@ -155,6 +156,12 @@ struct DecodeArgs {
 cudaError_t launch_decode(const DecodeLayout &L, const DecodeArgs &a, int32_t num_blocks_pool,
                           cudaStream_t stream, Tracer *tr);
 
+// Bit copy of n blocks (device ids) between a pool's caches and a staging
+// buffer [n][K, V][Hkv][16][d] (transfer.cu).
+cudaError_t launch_block_copy(const int32_t *ids, int32_t n, int32_t Hkv, int32_t d, void *k_cache,
+                              void *v_cache, void *staging, int32_t num_blocks, bool to_staging, int *err,
+                              int num_sms, cudaStream_t stream);
+
 struct PrefillArgs {
     const void *q;
     void *out;
@@ -170,6 +177,7 @@ struct PrefillArgs {
     const CUtensorMap *tmap_k;  // host copies, passed by value to the kernel
     const CUtensorMap *tmap_v;
     int *err;
+    const unsigned long long *tree_mask;   // null, or [T] draft masks (tree verification)
 };
 
 cudaError_t launch_prefill(const PrefillArgs &a, cudaStream_t stream, Tracer *tr);

@@ -98,6 +98,9 @@ struct KernelParams {
     int32_t parts_per_head;     // partial slots per (request, q head)
     float *o_part;              // [R*Hq*parts][D] unnormalised O
     float2 *ml_part;            // [R*Hq*parts] (running max (base 2), sum)
+    // suffix prefill only: null, or [T] draft masks (bit j of new token t's
+    // mask: t sees new token j of its request; at most 64 new tokens each)
+    const unsigned long long *tree_mask;
 };
 
 // Row maximum of the 128 raw scores a thread holds (8 independent chains).
@@ -155,7 +158,7 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
 //   item, key split); tile X row i = member X*tpt + i / g of the item; keys =
 //   the split's range of the group's prefix blocks (read through the first
 //   member's table row), all visible; writes unnormalised partials.
-template <int D, bool PREFIX>
+template <int D, bool PREFIX, bool TREE = false>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tile_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
                      const KernelParams p) {
@@ -465,6 +468,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int qi = x * p.tpt + row / p.g;         // query of the item behind this row
         // last visible key (item-local numbering of the key range)
         const int pos = (!PREFIX && valid) ? q_pos0 + qi : kv_end - 1;
+        // tree-shaped drafts: new token qi sees the request's new tokens whose
+        // bits are set in its mask (its ancestors and itself), all context keys
+        constexpr bool tree = !PREFIX && TREE;
+        const int new0 = q_pos0 - q0;                 // position of the request's first new token
+        const unsigned long long tmask = (tree && valid) ? __ldg(p.tree_mask + cu0 + q0 + qi) : ~0ull;
         const bool active = (x == 0) || has_b;
         float m = -INFINITY, l = 0.f;
         bool ok = active;
@@ -476,13 +484,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int c = 0; c < 4; ++c) tmem_ld32(s_addr + c * 32, sr[c]);
             tmem_wait_ld();
             const int lim = pos - j * kKeys;          // keys with column index <= lim are visible
-            const bool all_visible = __all_sync(0xffffffffu, lim >= kKeys - 1);
+            const int d0 = new0 - j * kKeys;          // column of the first new token (may be < 0)
+            const bool tree_tile = tree && d0 < kKeys;
+            const bool all_visible = __all_sync(0xffffffffu, lim >= kKeys - 1 && !tree_tile);
             if (!all_visible) {
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
 #pragma unroll
-                    for (int e = 0; e < 32; ++e)
-                        if (c * 32 + e > lim) sr[c][e] = __float_as_uint(-INFINITY);
+                    for (int e = 0; e < 32; ++e) {
+                        const int col = c * 32 + e;
+                        bool vis = col <= lim;
+                        // col - d0 <= pos - new0 < 64 whenever col <= lim
+                        if (vis && tree_tile && col >= d0) vis = (tmask >> (col - d0)) & 1ull;
+                        if (!vis) sr[c][e] = __float_as_uint(-INFINITY);
+                    }
             }
             // The first tile finds its row max before the pass.  Later tiles
             // compute P against the running max m, however stale: the same m
@@ -599,16 +614,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
-template <int D, bool PREFIX>
+template <int D, bool PREFIX, bool TREE = false>
 static cudaError_t launch_tile_kernel(dim3 grid, const CUtensorMap &tk, const CUtensorMap &tv,
                                       const KernelParams &p, cudaStream_t stream) {
     // the d = 64 tiles are smaller; ask for the d = 128 footprint anyway so
     // one CTA owns an SM (its 512 TMEM columns never wait on a neighbour)
     static SmemLimit limit;
-    cudaError_t e = limit.ensure(reinterpret_cast<const void *>(attn_tile_kernel<D, PREFIX>),
+    cudaError_t e = limit.ensure(reinterpret_cast<const void *>(attn_tile_kernel<D, PREFIX, TREE>),
                                  Layout<128>::kDynSmem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(attn_tile_kernel<D, PREFIX>, grid, dim3(kThreads), Layout<128>::kDynSmem, stream,
+    return launch_pdl(attn_tile_kernel<D, PREFIX, TREE>, grid, dim3(kThreads), Layout<128>::kDynSmem, stream,
                       tk, tv, p);
 }
 
@@ -626,13 +641,19 @@ cudaError_t launch_prefill(const PrefillArgs &a, cudaStream_t stream, Tracer *tr
     p.num_blocks_pool = a.num_blocks_pool;
     p.scale_log2 = a.scale_log2;
     p.err = a.err;
+    p.tree_mask = a.tree_mask;
     const int items = (a.max_seqlen_q + 2 * p.tpt - 1) / (2 * p.tpt);
     if (items <= 0 || a.R <= 0) return cudaSuccess;
     if (items > 65535) return cudaErrorInvalidConfiguration;
     dim3 grid((unsigned)(a.R * a.Hkv), (unsigned)items);
     if (tr) tr->begin(kKernelPrefill, stream);
-    cudaError_t e = a.d == 128 ? launch_tile_kernel<128, false>(grid, *a.tmap_k, *a.tmap_v, p, stream)
-                               : launch_tile_kernel<64, false>(grid, *a.tmap_k, *a.tmap_v, p, stream);
+    cudaError_t e;
+    if (p.tree_mask)
+        e = a.d == 128 ? launch_tile_kernel<128, false, true>(grid, *a.tmap_k, *a.tmap_v, p, stream)
+                       : launch_tile_kernel<64, false, true>(grid, *a.tmap_k, *a.tmap_v, p, stream);
+    else
+        e = a.d == 128 ? launch_tile_kernel<128, false>(grid, *a.tmap_k, *a.tmap_v, p, stream)
+                       : launch_tile_kernel<64, false>(grid, *a.tmap_k, *a.tmap_v, p, stream);
     if (tr) tr->end(kKernelPrefill, stream);
     return e;
 }

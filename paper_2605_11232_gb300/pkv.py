@@ -43,6 +43,8 @@ EXPORTS = [
     "pkv_prefix_cache_destroy", "pkv_prefix_cache_match", "pkv_prefix_cache_insert",
     "pkv_prefix_cache_evict", "pkv_prefix_cache_size", "pkv_prefix_groups_build",
     "pkv_selftest_wait_timeout", "pkv_lora_dispatch", "pkv_check_block_table",
+    "paged_attn_verify_tree", "pkv_tree_masks", "pkv_blocks_staging_size", "pkv_blocks_gather",
+    "pkv_blocks_scatter",
 ]
 
 
@@ -75,7 +77,10 @@ class StepLayout(ctypes.Structure):
     """Byte offsets of one decode step's inputs in a packed buffer (pkv_step_layout)."""
     _fields_ = [("q", ctypes.c_size_t), ("k_new", ctypes.c_size_t), ("v_new", ctypes.c_size_t),
                 ("slot_mapping", ctypes.c_size_t), ("context_lens", ctypes.c_size_t),
-                ("bytes", ctypes.c_size_t)]
+                ("bytes", ctypes.c_size_t), ("flags", ctypes.c_uint64)]
+
+
+PKV_STEP_FUSED_WRITE = 1
 
 
 _lib = None
@@ -127,6 +132,11 @@ def load(path: str | None = None):
         "pkv_selftest_wait_timeout": [V, i32, V],
         "pkv_lora_dispatch": [P, P, i32, P, i32, i32, P, P, P, P, P],
         "pkv_check_block_table": [V, P, i32, i32, P, P],
+        "paged_attn_verify_tree": [V, V, V, V, V, V, V, i32, i32, i32, i32, f32, V, V],
+        "pkv_tree_masks": [P, P, i32, P],
+        "pkv_blocks_staging_size": [V, i32, ctypes.POINTER(sz)],
+        "pkv_blocks_gather": [V, V, i32, V, V],
+        "pkv_blocks_scatter": [V, V, i32, V, V],
         "pkv_trace_read": [V, P, i32, P],
     }
     for name, args in sig.items():
@@ -354,6 +364,61 @@ def paged_attn_prefill(pool, q, out, lse, cu_seqlens_q, context_lens, block_tabl
         pool, _dptr(q), _dptr(out), _dptr(lse), _dptr(cu_seqlens_q), _dptr(context_lens),
         _dptr(block_table), int(block_table.shape[1]), int(context_lens.shape[0]),
         int(max_seqlen_q), int(q.shape[1]), float(scale), _stream(stream)))
+
+
+def paged_attn_verify_tree(pool, q, out, lse, cu_seqlens_q, context_lens, block_table,
+                           max_seqlen_q: int, scale: float, tree_mask, stream=None):
+    """paged_attn_prefill over tree-shaped drafts: tree_mask is a device
+    int64 tensor [T] of draft masks (pkv_tree_masks)."""
+    import torch
+    _check_attn_args(pool, q, out, lse, context_lens, block_table, 0)
+    _need(tuple(out.shape) == tuple(q.shape), lambda: f"out must have q's shape {list(q.shape)}")
+    cs = _check_tensor("cu_seqlens_q", cu_seqlens_q, torch.int32, 1)
+    _need(cs[0] == context_lens.shape[0] + 1,
+          lambda: f"cu_seqlens_q must have {context_lens.shape[0] + 1} entries")
+    ms = _check_tensor("tree_mask", tree_mask, torch.int64, 1)
+    _need(ms[0] >= q.shape[0], lambda: f"tree_mask has {ms[0]} entries for {q.shape[0]} rows")
+    _check(load().paged_attn_verify_tree(
+        pool, _dptr(q), _dptr(out), _dptr(lse), _dptr(cu_seqlens_q), _dptr(context_lens),
+        _dptr(block_table), int(block_table.shape[1]), int(context_lens.shape[0]),
+        int(max_seqlen_q), int(q.shape[1]), float(scale), _dptr(tree_mask), _stream(stream)))
+
+
+def pkv_blocks_staging_size(pool, n: int) -> int:
+    out = ctypes.c_size_t(0)
+    _check(load().pkv_blocks_staging_size(pool, int(n), ctypes.byref(out)))
+    return int(out.value)
+
+
+def _check_transfer_args(pool, block_ids, staging):
+    import torch
+    n = _check_tensor("block_ids", block_ids, torch.int32, 1)[0]
+    nbytes = staging.numel() * staging.element_size()
+    need = pkv_blocks_staging_size(pool, n)
+    _need(staging.is_cuda and staging.is_contiguous() and nbytes >= need,
+          lambda: f"staging must be a contiguous device buffer of >= {need} bytes, got {nbytes}")
+    return n
+
+
+def pkv_blocks_gather(pool, block_ids, staging, stream=None):
+    """Copy the pool's blocks block_ids (device int32 [n]) into staging."""
+    n = _check_transfer_args(pool, block_ids, staging)
+    _check(load().pkv_blocks_gather(pool, _dptr(block_ids), n, _dptr(staging), _stream(stream)))
+
+
+def pkv_blocks_scatter(pool, block_ids, staging, stream=None):
+    """Copy staging into the pool's blocks block_ids (device int32 [n])."""
+    n = _check_transfer_args(pool, block_ids, staging)
+    _check(load().pkv_blocks_scatter(pool, _dptr(block_ids), n, _dptr(staging), _stream(stream)))
+
+
+def pkv_tree_masks(parent, cu_seqlens) -> np.ndarray:
+    """Draft masks (int64 view of the uint64 bits) of tree-shaped drafts."""
+    par = np.ascontiguousarray(parent, np.int32)
+    cu = np.ascontiguousarray(cu_seqlens, np.int32)
+    out = np.zeros(max(len(par), 1), np.uint64)
+    _check(load().pkv_tree_masks(_np_ptr(par), _np_ptr(cu), len(cu) - 1, _np_ptr(out)))
+    return out[:len(par)].view(np.int64)
 
 
 def make_prefix_groups(num_groups=0, max_group_blocks=0, max_group_members=0, group_start=None,

@@ -309,16 +309,18 @@ def test_decode_short_and_ragged_segments(groups):
     b.close()
 
 
+@pytest.mark.parametrize("fused", [False, True])
 @pytest.mark.parametrize("groups", [False, True])
-def test_decode_step_from_host_buffers_bit_exact(groups):
+def test_decode_step_from_host_buffers_bit_exact(groups, fused):
     """paged_attn_decode_step (one H2D copy of the packed inputs, cache write,
-    decode, D2H copy of the output) gives the bits of kv_cache_write +
-    paged_attn_decode on device inputs, on two steps in a row."""
+    decode, D2H copy of the output; fused: the decode kernels store the new
+    tokens) gives the bits of kv_cache_write + paged_attn_decode on device
+    inputs, on two steps in a row."""
     need_gpu()
     w = make_workload("l8b_decode", scale_requests=0.25)
     b = B.build_batch(w, poison=True)
     ref, ref_lse = run_decode(b, use_groups=groups)
-    layout, hosts, dev = B.step_buffers(b, copies=1)
+    layout, hosts, dev = B.step_buffers(b, copies=1, fused=fused)
     R = b.dec.stop - b.dec.start
     ws = B.decode_workspace(b, groups)
     out = torch.empty_like(ref)
@@ -340,7 +342,7 @@ def test_decode_step_from_host_buffers_bit_exact(groups):
     torch.cuda.synchronize()
     bad = pkv.StepLayout(q=layout.q, k_new=layout.k_new + 8, v_new=layout.v_new,
                          slot_mapping=layout.slot_mapping, context_lens=layout.context_lens,
-                         bytes=layout.bytes)
+                         bytes=layout.bytes, flags=layout.flags)
     with pytest.raises(pkv.PkvError) as e:
         pkv.paged_attn_decode_step(b.pool, hosts[0], dev, bad, w.num_new_tokens, b.table[b.dec],
                                    w.num_q_heads, w.scale, None, ws, out)
