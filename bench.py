@@ -515,6 +515,57 @@ def measure_transfer(steps, warmup):
                     "of the staging buffer is not measured)"}
 
 
+def measure_lora(steps, warmup):
+    """Segmented multi-adapter LoRA projection (Sec. 5.6): Llama-3-8B-shaped
+    projection (4096 x 4096), rank-16 adapters.  Case C1: the 12-prompt
+    4/3/3/2 request over four adapters, batched by pkv_lora_dispatch
+    (adapter first, length buckets at 1024 / 2048 tokens); and a larger
+    synthetic request (64 prompts, 8 adapters, a quarter base-only).
+    TFLOP/s on the base and low-rank products; cuBLAS's base GEMM alone
+    (torch.matmul, bf16) on the same rows beside it, for context."""
+    import numpy as np
+    import torch
+
+    from paper_2605_11232_gb300 import pkv
+
+    def one(lens, ads, n_ad, seed):
+        # base-only prompts are dispatched as adapter n_ad (their own group)
+        # and run with no adapter (-1)
+        order, batches = pkv.pkv_lora_dispatch(np.array([a if a >= 0 else n_ad for a in ads], np.int32),
+                                               np.array(lens, np.int32), np.array([1024, 2048], np.int32), 0)
+        starts, badapter = [0], []
+        for adapter, _bk, b0, b1 in batches:
+            starts.append(starts[-1] + sum(lens[order[i]] for i in range(b0, b1)))
+            badapter.append(adapter if adapter < n_ad else -1)
+        T, d, r = starts[-1], 4096, 16
+        g = torch.Generator(device="cuda").manual_seed(seed)
+        x = torch.randn((T, d), device="cuda", generator=g).to(torch.bfloat16)
+        w = (torch.randn((d, d), device="cuda", generator=g) / d ** 0.5).to(torch.bfloat16)
+        a = (torch.randn((n_ad, r, d), device="cuda", generator=g) / d ** 0.5).to(torch.bfloat16)
+        b = (torch.randn((n_ad, d, r), device="cuda", generator=g) / r ** 0.5).to(torch.bfloat16)
+        scale = np.full(n_ad, 2.0, np.float32)
+        y = torch.empty((T, d), dtype=torch.bfloat16, device="cuda")
+        flush_buf = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device="cuda")
+        step = lambda: pkv.pkv_lora_sgmv(x, w, a, b, scale, starts, badapter, y)
+        ms = _timed(step, lambda: flush_buf.fill_(1), steps, warmup, torch.cuda.current_stream())
+        t_lora = sum(starts[k + 1] - starts[k] for k in range(len(badapter)) if badapter[k] >= 0)
+        flops = 2 * T * d * d + 2 * t_lora * (d * r + r * d)
+        base = _timed(lambda: torch.matmul(x, w.t()), lambda: flush_buf.fill_(1), steps, warmup,
+                      torch.cuda.current_stream())
+        mean, bmean = statistics.mean(ms), statistics.mean(base)
+        return {"tokens": T, "segments": len(badapter), "adapters": n_ad, "rank": r,
+                "ms_per_call": mean, "tflops": flops / (mean * 1e-3) / 1e12,
+                "cublas_base_only_ms": bmean, "cublas_base_only_tflops": 2 * T * d * d / (bmean * 1e-3) / 1e12}
+
+    c1 = one([412, 1830, 2650, 977, 1210, 2205, 388, 1499, 2800, 640, 1750, 2120],
+             [0, 0, 0, 0, 1, 1, 1, 2, 2, 2, 3, 3], 4, 11)
+    rng = np.random.default_rng(12)
+    lens = rng.integers(300, 2900, 64).tolist()
+    ads = [int(v) if v < 8 else -1 for v in rng.integers(0, 11, 64)]
+    big = one(lens, ads, 8, 12)
+    return {"case_c1": c1, "synthetic_64": big}
+
+
 def summarize(res, peaks):
     hbm, tf_burst, tf_sust, kind = peaks
     ms = statistics.mean(res["step_ms"])
@@ -656,6 +707,11 @@ def main():
     from paper_2605_11232_gb300 import pkv
     pkv.load()
     peaks = load_peaks()
+    if args.profile in ("lora_sgmv", "pd_block_transfer", "spec_verify_tree"):
+        fn = {"lora_sgmv": measure_lora, "pd_block_transfer": measure_transfer,
+              "spec_verify_tree": measure_verify}[args.profile]
+        print(json.dumps({"profile": args.profile, **fn(args.steps, args.warmup)}), flush=True)
+        return 0
     if args.profile:
         r = measure_workload(args.profile, args.steps, args.warmup)
         print(json.dumps({"profile": args.profile, **summarize(r, peaks)}), flush=True)
@@ -674,11 +730,15 @@ def main():
                 extra[name] = summarize(r, peaks)
             except Exception as e:   # report, do not hide
                 extra[name] = {"error": str(e)}
-        for name, fn in (("spec_verify_tree", measure_verify), ("pd_block_transfer", measure_transfer)):
+        for name, fn in (("spec_verify_tree", measure_verify), ("pd_block_transfer", measure_transfer),
+                         ("lora_sgmv", measure_lora)):
             try:
                 r = fn(max(10, args.steps // 10), 3)
                 if "transfer_hbm_gbs" in r:
                     r["frac_of_measured_hbm"] = r["transfer_hbm_gbs"] / peaks[0]
+                for sub in ("case_c1", "synthetic_64"):
+                    if sub in r:
+                        r[sub]["frac_of_measured_bf16"] = r[sub]["tflops"] / peaks[1]
                 if "verify_tflops" in r:
                     r["verify_frac_of_measured_bf16"] = r["verify_tflops"] / peaks[1]
                     r["step_frac_of_measured_hbm"] = r["step_hbm_gbs"] / peaks[0]

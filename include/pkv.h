@@ -274,6 +274,37 @@ int pkv_lora_dispatch(const int32_t *adapter_id, const int32_t *prompt_len, int3
                       int32_t *order_out, int32_t *batch_start_out, int32_t *batch_adapter_out,
                       int32_t *batch_bucket_out, int32_t *n_batches_out);
 
+/* ---- multi-adapter LoRA projection (device) ---------------------------------- */
+
+/* The segmented multi-adapter LoRA projection of Sec. 5.6 (one base model,
+ * several adapters, a mixed request run as the per-adapter batches of
+ * pkv_lora_dispatch): for the tokens t of segment s with adapter
+ * a = seg_adapter[s],
+ *     y_t = W x_t + scale[a] * B_a (A_a x_t)     (a = -1: y_t = W x_t).
+ * The paper names LoRA adapters but prints no formula; this is the standard
+ * low-rank update.  Both products run on the tensor cores in one kernel (bf16
+ * operands, fp32 accumulation); A_a x_t is scaled and rounded to bf16 before
+ * its product with B_a; y is rounded to bf16.
+ *  x: device bf16 [num_tokens][d_in]; w: device bf16 [d_out][d_in];
+ *  lora_a: device bf16 [num_adapters][rank][d_in];
+ *  lora_b: device bf16 [num_adapters][d_out][rank];
+ *  y: device bf16 [num_tokens][d_out]; all 16-byte aligned.
+ *  scale: host float [num_adapters]; seg_start: host int32 [num_segments + 1]
+ *  from 0 to num_tokens, non-decreasing; seg_adapter: host int32
+ *  [num_segments], each in [-1, num_adapters).
+ *  error_word: device int32 the kernel latches DEVICE_TIMEOUT into if a
+ *  bounded wait runs out (may be NULL).
+ * Limits: d_in a multiple of 64, d_out of 256, rank 16, 32, 48 or 64
+ * (UNSUPPORTED otherwise); each segment is cut into 128-row tiles, at most
+ * PKV_LORA_MAX_TILES per call (UNSUPPORTED beyond: split the call).
+ * Errors: INVALID_ARG, UNSUPPORTED, CUDA. */
+#define PKV_LORA_MAX_TILES 1024
+int pkv_lora_sgmv(const void *x, const void *w, const void *lora_a, const void *lora_b,
+                  const float *scale, const int32_t *seg_start, const int32_t *seg_adapter,
+                  int32_t num_segments, int32_t num_tokens, int32_t d_in, int32_t d_out,
+                  int32_t rank, int32_t num_adapters, void *y, int32_t *error_word,
+                  pkv_stream_t stream);
+
 /* ---- a3: cache write (device) ------------------------------------------- */
 
 /* Scatter new-token keys and values into their slots (bit-exact copy).

@@ -19,7 +19,7 @@ OUT = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT, "libpkv.so")
 ROOT = os.path.dirname(HERE)
 SOURCES = ["pkv_api.cpp", "prefix_cache.cpp", "lora_dispatch.cpp", "cache_write.cu", "decode.cu", "prefill.cu",
-           "decode_noalloc.cu", "selftest.cu", "transfer.cu"]
+           "decode_noalloc.cu", "selftest.cu", "transfer.cu", "lora.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
               "--expt-relaxed-constexpr", "-I", os.path.join(ROOT, "include")]

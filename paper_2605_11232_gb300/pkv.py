@@ -44,7 +44,7 @@ EXPORTS = [
     "pkv_prefix_cache_evict", "pkv_prefix_cache_size", "pkv_prefix_groups_build",
     "pkv_selftest_wait_timeout", "pkv_lora_dispatch", "pkv_check_block_table",
     "paged_attn_verify_tree", "pkv_tree_masks", "pkv_blocks_staging_size", "pkv_blocks_gather",
-    "pkv_blocks_scatter",
+    "pkv_blocks_scatter", "pkv_lora_sgmv",
 ]
 
 
@@ -135,6 +135,7 @@ def load(path: str | None = None):
         "paged_attn_verify_tree": [V, V, V, V, V, V, V, i32, i32, i32, i32, f32, V, V],
         "pkv_tree_masks": [P, P, i32, P],
         "pkv_blocks_staging_size": [V, i32, ctypes.POINTER(sz)],
+        "pkv_lora_sgmv": [V, V, V, V, P, P, P, i32, i32, i32, i32, i32, i32, V, V, V],
         "pkv_blocks_gather": [V, V, i32, V, V],
         "pkv_blocks_scatter": [V, V, i32, V, V],
         "pkv_trace_read": [V, P, i32, P],
@@ -410,6 +411,32 @@ def pkv_blocks_scatter(pool, block_ids, staging, stream=None):
     """Copy staging into the pool's blocks block_ids (device int32 [n])."""
     n = _check_transfer_args(pool, block_ids, staging)
     _check(load().pkv_blocks_scatter(pool, _dptr(block_ids), n, _dptr(staging), _stream(stream)))
+
+
+def pkv_lora_sgmv(x, w, lora_a, lora_b, scale, seg_start, seg_adapter, y, error_word=None,
+                  stream=None):
+    """y = W x + s_a B_a (A_a x) per segment (device bf16 tensors; scale,
+    seg_start, seg_adapter host arrays)."""
+    import torch
+    T, d_in = _check_tensor("x", x, torch.bfloat16, 2)
+    d_out, wi = _check_tensor("w", w, torch.bfloat16, 2)
+    _need(wi == d_in, lambda: f"w must be [d_out][{d_in}], got {list(w.shape)}")
+    n_ad, rank, ai = _check_tensor("lora_a", lora_a, torch.bfloat16, 3)
+    _need(ai == d_in, lambda: f"lora_a must be [n][rank][{d_in}], got {list(lora_a.shape)}")
+    bs = _check_tensor("lora_b", lora_b, torch.bfloat16, 3)
+    _need(tuple(bs) == (n_ad, d_out, rank), lambda: f"lora_b must be [{n_ad}][{d_out}][{rank}], got {list(bs)}")
+    ys = _check_tensor("y", y, torch.bfloat16, 2)
+    _need(tuple(ys) == (T, d_out), lambda: f"y must be [{T}][{d_out}], got {list(ys)}")
+    for name, t in (("x", x), ("w", w), ("lora_a", lora_a), ("lora_b", lora_b), ("y", y)):
+        _need(t.is_cuda and t.is_contiguous(), lambda: f"{name} must be a contiguous device tensor")
+    sc = np.ascontiguousarray(scale, np.float32)
+    st = np.ascontiguousarray(seg_start, np.int32)
+    sa = np.ascontiguousarray(seg_adapter, np.int32)
+    _need(len(sc) >= n_ad, lambda: f"scale needs {n_ad} entries")
+    _need(len(st) == len(sa) + 1, "seg_start must have one entry more than seg_adapter")
+    _check(load().pkv_lora_sgmv(_dptr(x), _dptr(w), _dptr(lora_a), _dptr(lora_b), _np_ptr(sc), _np_ptr(st),
+                                _np_ptr(sa), len(sa), int(T), int(d_in), int(d_out), int(rank), int(n_ad),
+                                _dptr(y), _dptr(error_word), _stream(stream)))
 
 
 def pkv_tree_masks(parent, cu_seqlens) -> np.ndarray:
