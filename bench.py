@@ -275,16 +275,14 @@ def measure_workload(name, steps, warmup, use_groups=True, e2e_steps=0):
     def flush():
         flush_buf.fill_(1)
 
-    rows_w = rows_p   # tokens the write kernel stores: the prefill subset's
-    fused_bytes = write_bytes(w, w.num_new_tokens - (rows_w.stop - rows_w.start))
+    # every new token's K/V is stored by the attention kernel that reads it:
+    # the prefill subset's by the prefill kernel (paged_attn_prefill_append),
+    # the decode subset's by the decode split pass (paged_attn_decode_append)
+    fused_bytes = write_bytes(w, w.num_new_tokens - (rows_p.stop - rows_p.start))
 
     def step():
-        # the prefill subset's new tokens by kv_cache_write, then its
-        # attention; the decode subset's own K/V are stored by the decode
-        # kernels themselves (paged_attn_decode_append)
         if Rp:
-            pkv.kv_cache_write(b.pool, b.k_new[rows_w], b.v_new[rows_w], b.slots[rows_w])
-            B.run_prefill(b, out_p, None)
+            B.run_prefill_append(b, out_p, None)
         if Rd:
             B.run_decode_append(b, out_d, None, ws, groups_ok)
 
@@ -320,7 +318,7 @@ def measure_workload(name, steps, warmup, use_groups=True, e2e_steps=0):
     pkv.pkv_trace_enable(b.pool, False)
     assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
     # algorithmic bytes each decode kernel is responsible for
-    kb = {"kv_cache_write": write_bytes(w, rows_w.stop - rows_w.start)}
+    kb = {}
     if Rd:
         rows_priv = sum(int(w.context_lens[r]) - w.prefix_len_of(r) for r in range(b.dec.start, b.dec.stop))
         used = {int(w.group_of_req[r]) for r in range(b.dec.start, b.dec.stop)} - {-1}

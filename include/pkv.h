@@ -340,6 +340,26 @@ int paged_attn_prefill(pkv_pool_t pool, const void *q, void *out, float *lse,
                        int32_t max_seqlen_q, int32_t num_q_heads, float scale,
                        pkv_stream_t stream);
 
+/* paged_attn_prefill with the cache write of the new tokens fused in (Sec.
+ * 5.4: only the new tokens cost anything once the prefix is cached): new
+ * token i of request r is stored into its slot (position
+ * context_lens[r] - n_r + i, through block_table) by the prefill kernel, and
+ * the new keys and values are read from k_new / v_new while attending.  The
+ * outputs, and the pool afterwards, equal kv_cache_write of those tokens
+ * followed by paged_attn_prefill.
+ *  k_new, v_new: device bf16 [num_new_tokens][num_kv_heads][head_dim],
+ *  16-byte aligned, rows in q's order (num_new_tokens = cu_seqlens_q[R]).
+ *  Each request's cached part, context_lens[r] - n_r, must be whole blocks (a
+ *  multiple of 16, as prefix caching leaves it): a request that is not is
+ *  skipped and latches DEVICE_BOUNDS.  The blocks of the new tokens must be
+ *  the request's own (reference count 1).
+ * Every other argument and the errors are those of paged_attn_prefill. */
+int paged_attn_prefill_append(pkv_pool_t pool, const void *q, const void *k_new, const void *v_new,
+                              int32_t num_new_tokens, void *out, float *lse, const int32_t *cu_seqlens_q,
+                              const int32_t *context_lens, const int32_t *block_table, int32_t max_blocks,
+                              int32_t num_requests, int32_t max_seqlen_q, int32_t num_q_heads, float scale,
+                              pkv_stream_t stream);
+
 /* ---- speculative-decode verification with tree-shaped drafts (device) ---- */
 
 /* paged_attn_prefill where each request's new tokens are draft tokens of a

@@ -245,6 +245,14 @@ def run_prefill(b: Batch, out: torch.Tensor, lse, stream=None):
                            b.table[b.pre], b.max_seqlen_pre, b.w.scale, stream)
 
 
+def run_prefill_append(b: Batch, out: torch.Tensor, lse, stream=None):
+    """The prefill subset's cache write and attention in one call: the
+    prefill kernel stores each new token's K/V."""
+    rows = new_token_rows(b.w, b.pre)
+    pkv.paged_attn_prefill_append(b.pool, b.q[rows], b.k_new[rows], b.v_new[rows], out, lse, b.cu_pre,
+                                  b.context_lens[b.pre], b.table[b.pre], b.max_seqlen_pre, b.w.scale, stream)
+
+
 def kv_waste(b: Batch) -> float:
     """Fraction of allocated KV slots holding no token, shared blocks once."""
     used_blocks = b.num_blocks_pool - pkv.kv_pool_num_free(b.pool)

@@ -433,10 +433,32 @@ int kv_cache_write(pkv_pool_t pool, const void *k_new, const void *v_new,
 namespace {
 
 // paged_attn_prefill, with tree-shaped draft masks when tree_mask is set
+// TMA descriptor of new-token rows [T][Hkv][d] (k_new or v_new): a 3-D view
+// {d, Hkv, T}, box {64, 1, 16} = 16 tokens of one kv head, laid out in shared
+// memory exactly like a pool box of 16 slots (128-byte swizzle).
+int new_rows_tmap(CUtensorMap *m, const void *base, int32_t T, int32_t Hkv, int32_t d) {
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn)
+        return fail(PKV_ERR_CUDA, "cuTensorMapEncodeTiled entry point not found");
+    auto encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    cuuint64_t dims[3] = {(cuuint64_t)d, (cuuint64_t)Hkv, (cuuint64_t)T};
+    cuuint64_t strides[2] = {(cuuint64_t)d * 2, (cuuint64_t)d * 2 * Hkv};
+    cuuint32_t box[3] = {64, 1, 16};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box,
+                        estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(PKV_ERR_CUDA, "cuTensorMapEncodeTiled (new rows) failed (%d)", (int)r);
+    return PKV_OK;
+}
+
 int prefill_impl(pkv_pool_t pool, const void *q, void *out, float *lse, const int32_t *cu_seqlens_q,
                  const int32_t *context_lens, const int32_t *block_table, int32_t max_blocks,
                  int32_t num_requests, int32_t max_seqlen_q, int32_t num_q_heads, float scale,
-                 const uint64_t *tree_mask, pkv_stream_t stream) {
+                 const uint64_t *tree_mask, const void *k_new, const void *v_new, int32_t num_new_tokens,
+                 pkv_stream_t stream) {
     int rc = check_kernel_pool(pool);
     if (rc != PKV_OK) return rc;
     const pkv_pool_desc &d = pool->desc;
@@ -454,8 +476,17 @@ int prefill_impl(pkv_pool_t pool, const void *q, void *out, float *lse, const in
     if (!q || !out || !cu_seqlens_q || !context_lens || !block_table)
         return fail(PKV_ERR_INVALID_ARG, "NULL buffer");
     if (!aligned16(q) || !aligned16(out)) return fail(PKV_ERR_INVALID_ARG, "misaligned q/out");
+    if ((k_new == nullptr) != (v_new == nullptr)) return fail(PKV_ERR_INVALID_ARG, "give both k_new and v_new");
+    if (k_new && (!aligned16(k_new) || !aligned16(v_new)))
+        return fail(PKV_ERR_INVALID_ARG, "misaligned k_new/v_new");
+    if (k_new && num_new_tokens <= 0) return fail(PKV_ERR_INVALID_ARG, "num_new_tokens must be positive");
     if ((rc = set_device(pool)) != PKV_OK) return rc;
     if ((rc = build_tmaps(pool)) != PKV_OK) return rc;
+    CUtensorMap tkn, tvn;
+    if (k_new) {
+        if ((rc = new_rows_tmap(&tkn, k_new, num_new_tokens, d.num_kv_heads, d.head_dim)) != PKV_OK) return rc;
+        if ((rc = new_rows_tmap(&tvn, v_new, num_new_tokens, d.num_kv_heads, d.head_dim)) != PKV_OK) return rc;
+    }
     pkv::PrefillArgs a{};
     a.q = q; a.out = out; a.lse = lse;
     a.cu_seqlens_q = cu_seqlens_q; a.context_lens = context_lens;
@@ -467,6 +498,11 @@ int prefill_impl(pkv_pool_t pool, const void *q, void *out, float *lse, const in
     a.tmap_k = &pool->tmap_k; a.tmap_v = &pool->tmap_v;
     a.err = pool->d_err;
     a.tree_mask = reinterpret_cast<const unsigned long long *>(tree_mask);
+    if (k_new) {
+        a.k_new = k_new; a.v_new = v_new;
+        a.k_cache = pool->k_cache; a.v_cache = pool->v_cache;
+        a.tmap_kn = &tkn; a.tmap_vn = &tvn;
+    }
     cudaError_t e = pkv::launch_prefill(a, static_cast<cudaStream_t>(stream), pool->tracer);
     if (e != cudaSuccess) return cuda_fail(e, "paged_attn_prefill launch");
     return ok();
@@ -482,7 +518,19 @@ int paged_attn_prefill(pkv_pool_t pool, const void *q, void *out, float *lse,
                        int32_t max_seqlen_q, int32_t num_q_heads, float scale,
                        pkv_stream_t stream) {
     return prefill_impl(pool, q, out, lse, cu_seqlens_q, context_lens, block_table, max_blocks,
-                        num_requests, max_seqlen_q, num_q_heads, scale, nullptr, stream);
+                        num_requests, max_seqlen_q, num_q_heads, scale, nullptr, nullptr, nullptr, 0, stream);
+}
+
+int paged_attn_prefill_append(pkv_pool_t pool, const void *q, const void *k_new, const void *v_new,
+                              int32_t num_new_tokens, void *out, float *lse, const int32_t *cu_seqlens_q,
+                              const int32_t *context_lens, const int32_t *block_table, int32_t max_blocks,
+                              int32_t num_requests, int32_t max_seqlen_q, int32_t num_q_heads, float scale,
+                              pkv_stream_t stream) {
+    if (num_requests > 0 && max_seqlen_q > 0 && (!k_new || !v_new))
+        return fail(PKV_ERR_INVALID_ARG, "NULL k_new/v_new");
+    return prefill_impl(pool, q, out, lse, cu_seqlens_q, context_lens, block_table, max_blocks,
+                        num_requests, max_seqlen_q, num_q_heads, scale, nullptr, k_new, v_new, num_new_tokens,
+                        stream);
 }
 
 int paged_attn_verify_tree(pkv_pool_t pool, const void *q, void *out, float *lse,
@@ -495,7 +543,7 @@ int paged_attn_verify_tree(pkv_pool_t pool, const void *q, void *out, float *lse
         (!tree_mask || (reinterpret_cast<uintptr_t>(tree_mask) & 7)))
         return fail(PKV_ERR_INVALID_ARG, "tree_mask must be a non-NULL, 8-byte aligned device array");
     return prefill_impl(pool, q, out, lse, cu_seqlens_q, context_lens, block_table, max_blocks,
-                        num_requests, max_seqlen_q, num_q_heads, scale, tree_mask, stream);
+                        num_requests, max_seqlen_q, num_q_heads, scale, tree_mask, nullptr, nullptr, 0, stream);
 }
 
 int pkv_tree_masks(const int32_t *parent, const int32_t *cu_seqlens, int32_t num_requests,

@@ -178,6 +178,11 @@ struct PrefillArgs {
     const CUtensorMap *tmap_v;
     int *err;
     const unsigned long long *tree_mask;   // null, or [T] draft masks (tree verification)
+    // the new tokens' K/V stored by the kernel (null: already in the cache)
+    const void *k_new, *v_new;             // [T][Hkv][d]
+    void *k_cache, *v_cache;
+    const CUtensorMap *tmap_kn;            // 3-D maps over k_new / v_new
+    const CUtensorMap *tmap_vn;
 };
 
 cudaError_t launch_prefill(const PrefillArgs &a, cudaStream_t stream, Tracer *tr);

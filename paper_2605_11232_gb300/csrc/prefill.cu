@@ -101,6 +101,12 @@ struct KernelParams {
     // suffix prefill only: null, or [T] draft masks (bit j of new token t's
     // mask: t sees new token j of its request; at most 64 new tokens each)
     const unsigned long long *tree_mask;
+    // suffix prefill with the new tokens' K/V fused in: keys at positions
+    // >= L - n_r come from k_new / v_new (tensor maps tmkn / tmvn), and each
+    // CTA stores its own queries' K/V rows into the pool
+    int32_t fused;
+    const uint16_t *k_new, *v_new;   // [T][Hkv][D]
+    uint16_t *k_cache, *v_cache;     // the pool
 };
 
 // Row maximum of the 128 raw scores a thread holds (8 independent chains).
@@ -158,9 +164,10 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
 //   item, key split); tile X row i = member X*tpt + i / g of the item; keys =
 //   the split's range of the group's prefix blocks (read through the first
 //   member's table row), all visible; writes unnormalised partials.
-template <int D, bool PREFIX, bool TREE = false>
+template <int D, bool PREFIX, bool TREE = false, bool FUSED = false>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tile_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
+                     const __grid_constant__ CUtensorMap tmkn, const __grid_constant__ CUtensorMap tmvn,
                      const KernelParams p) {
     using Ly = Layout<D>;
     pdl_wait();
@@ -169,7 +176,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int h = blockIdx.x % p.Hkv;
-    int nq, nblk, kv_end, q_pos0 = 0, blk_off = 0, cu0 = 0, q0 = 0, m0 = 0;
+    int nq, nblk, kv_end, q_pos0 = 0, blk_off = 0, cu0 = 0, q0 = 0, m0 = 0, new_blk0 = 1 << 30, cached = 0;
     const int32_t *trow;
     if constexpr (!PREFIX) {
         const int r = blockIdx.x / p.Hkv;
@@ -183,6 +190,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (L < n_r || L > 16 * p.max_blocks) {
             if (threadIdx.x == 0) latch_error(p.err, kDevBounds);
             return;
+        }
+        cached = L - n_r;                 // keys before the request's new tokens
+        if constexpr (FUSED) {
+            // new keys come from k_new in whole 16-token blocks
+            if (cached & 15) {
+                if (threadIdx.x == 0) latch_error(p.err, kDevBounds);
+                return;
+            }
+            new_blk0 = cached >> 4;
         }
         q_pos0 = L - n_r + q0;            // absolute position of the item's first query
         kv_end = q_pos0 + nq;             // keys [0, kv_end) are visible to some row
@@ -288,15 +304,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t bar = sb + (k_side ? Ly::kKFull : Ly::kVFull) + 8 * s;
         const uint32_t dst = sb + (k_side ? Ly::kK0 : Ly::kV0) + s * Ly::kTile;
         mbar_arrive_expect_tx(bar, bytes);
-        for (int b = 0; b < nb; ++b)
+        // cached blocks from the pool; with the fused write, the request's
+        // new blocks (from new_blk0 on) from k_new / v_new, 16 tokens each
+        const int nb_pool = FUSED ? min(nb, max(0, new_blk0 - b0)) : nb;
+        for (int b = 0; b < nb_pool; ++b)
             for (int hf = 0; hf < Ly::kHalves; ++hf)
                 tma_load_4d(dst + hf * Ly::kHalfBytes + b * 2048, k_side ? &tmk : &tmv, hf * 64, 0, h,
                             blk_ids[b0 + b], bar);
+        if constexpr (FUSED) {
+            for (int b = nb_pool; b < nb; ++b)
+                for (int hf = 0; hf < Ly::kHalves; ++hf)
+                    tma_load_3d(dst + hf * Ly::kHalfBytes + b * 2048, k_side ? &tmkn : &tmvn, hf * 64, h,
+                                cu0 + (b0 + b) * 16 - cached, bar);
+        }
     };
     const int early = min(2, nkt);
     if (threadIdx.x == 0) {
         prefetch_tmap(&tmk);
         prefetch_tmap(&tmv);
+        if constexpr (FUSED) {
+            prefetch_tmap(&tmkn);
+            prefetch_tmap(&tmvn);
+        }
         for (int j = 0; j < early; ++j) {
             issue_kv(j, true);
             issue_kv(j, false);
@@ -370,6 +399,26 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (issued_k_only) {
                 const int j = issued_k_only - 1;
                 mbar_wait(sb + Ly::kKFull + 8 * (j & 1), (j >> 1) & 1, &quiet, kDrainLimitNs);
+            }
+            if constexpr (FUSED) {
+                // Whole blocks of the item's own new tokens are in the last
+                // two stages (an item has at most 64 tokens, so its blocks lie
+                // in the last two key tiles, whose stages are never reloaded):
+                // store them into the pool from there.  Blocks only partly
+                // the item's go by plain stores (warps 2-3).
+                if (!*abort && issued == nkt) {
+                    const int bfirst = (q_pos0 + 15) >> 4, blast = kv_end >> 4;   // [bfirst, blast)
+                    for (int bi = bfirst; bi < blast; ++bi) {
+                        const int j = bi >> 3, bb = bi & 7, st = j & 1;
+                        for (int hf = 0; hf < Ly::kHalves; ++hf) {
+                            const uint32_t off = st * Ly::kTile + hf * Ly::kHalfBytes + bb * 2048;
+                            tma_store_4d(&tmk, sb + Ly::kK0 + off, hf * 64, 0, h, blk_ids[bi]);
+                            tma_store_4d(&tmv, sb + Ly::kV0 + off, hf * 64, 0, h, blk_ids[bi]);
+                        }
+                    }
+                    bulk_commit();
+                    bulk_wait();
+                }
             }
         }
     } else if (warp == 1) {
@@ -454,6 +503,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_wait(sb + Ly::kDone, 0, &quiet, kDrainLimitNs);
         }
         __syncwarp();
+      } else if constexpr (FUSED) {
+        {
+            // ------------------------------------------------ store (warps 2-3)
+            // the K/V rows of this item's own queries (kv head h) that lie in
+            // blocks only partly the item's (the producer stores the whole
+            // ones by TMA); every new token belongs to exactly one item per head
+            constexpr int CPR = D / 8;
+            const int t0 = threadIdx.x - 64;
+            const int head_rows = min(nq, ((q_pos0 + 15) & ~15) - q_pos0);   // before the first whole block
+            const int tail0 = max(head_rows, (kv_end & ~15) - q_pos0);       // from the last partial block
+            const int n_plain = head_rows + (nq - tail0);
+            for (int i = t0; i < n_plain * 2 * CPR; i += 64) {
+                const int k = i / (2 * CPR), rem = i - k * 2 * CPR;
+                const int qi = k < head_rows ? k : tail0 + (k - head_rows);
+                const int isv = rem >= CPR, c = rem - isv * CPR;
+                const int pos = q_pos0 + qi;
+                const int64_t src = ((int64_t)(cu0 + q0 + qi) * p.Hkv + h) * D + c * 8;
+                const int64_t dst = (((int64_t)blk_ids[pos >> 4] * p.Hkv + h) * 16 + (pos & 15)) * D + c * 8;
+                const uint4 v = ldg_stream((isv ? p.v_new : p.k_new) + src);
+                *reinterpret_cast<uint4 *>((isv ? p.v_cache : p.k_cache) + dst) = v;
+            }
+        }
       }
     } else {
         // ------------------------------------------------------------ softmax
@@ -614,17 +685,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
-template <int D, bool PREFIX, bool TREE = false>
+template <int D, bool PREFIX, bool TREE = false, bool FUSED = false>
 static cudaError_t launch_tile_kernel(dim3 grid, const CUtensorMap &tk, const CUtensorMap &tv,
+                                      const CUtensorMap &tkn, const CUtensorMap &tvn,
                                       const KernelParams &p, cudaStream_t stream) {
     // the d = 64 tiles are smaller; ask for the d = 128 footprint anyway so
     // one CTA owns an SM (its 512 TMEM columns never wait on a neighbour)
     static SmemLimit limit;
-    cudaError_t e = limit.ensure(reinterpret_cast<const void *>(attn_tile_kernel<D, PREFIX, TREE>),
+    cudaError_t e = limit.ensure(reinterpret_cast<const void *>(attn_tile_kernel<D, PREFIX, TREE, FUSED>),
                                  Layout<128>::kDynSmem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(attn_tile_kernel<D, PREFIX, TREE>, grid, dim3(kThreads), Layout<128>::kDynSmem, stream,
-                      tk, tv, p);
+    return launch_pdl(attn_tile_kernel<D, PREFIX, TREE, FUSED>, grid, dim3(kThreads), Layout<128>::kDynSmem, stream,
+                      tk, tv, tkn, tvn, p);
 }
 
 cudaError_t launch_prefill(const PrefillArgs &a, cudaStream_t stream, Tracer *tr) {
@@ -642,18 +714,28 @@ cudaError_t launch_prefill(const PrefillArgs &a, cudaStream_t stream, Tracer *tr
     p.scale_log2 = a.scale_log2;
     p.err = a.err;
     p.tree_mask = a.tree_mask;
+    p.fused = a.k_new != nullptr;
+    p.k_new = static_cast<const uint16_t *>(a.k_new);
+    p.v_new = static_cast<const uint16_t *>(a.v_new);
+    p.k_cache = static_cast<uint16_t *>(a.k_cache);
+    p.v_cache = static_cast<uint16_t *>(a.v_cache);
+    // without the fused write the new-token maps are never read
+    const CUtensorMap &tkn = p.fused ? *a.tmap_kn : *a.tmap_k, &tvn = p.fused ? *a.tmap_vn : *a.tmap_v;
     const int items = (a.max_seqlen_q + 2 * p.tpt - 1) / (2 * p.tpt);
     if (items <= 0 || a.R <= 0) return cudaSuccess;
     if (items > 65535) return cudaErrorInvalidConfiguration;
     dim3 grid((unsigned)(a.R * a.Hkv), (unsigned)items);
     if (tr) tr->begin(kKernelPrefill, stream);
     cudaError_t e;
-    if (p.tree_mask)
-        e = a.d == 128 ? launch_tile_kernel<128, false, true>(grid, *a.tmap_k, *a.tmap_v, p, stream)
-                       : launch_tile_kernel<64, false, true>(grid, *a.tmap_k, *a.tmap_v, p, stream);
+    if (p.fused)
+        e = a.d == 128 ? launch_tile_kernel<128, false, false, true>(grid, *a.tmap_k, *a.tmap_v, tkn, tvn, p, stream)
+                       : launch_tile_kernel<64, false, false, true>(grid, *a.tmap_k, *a.tmap_v, tkn, tvn, p, stream);
+    else if (p.tree_mask)
+        e = a.d == 128 ? launch_tile_kernel<128, false, true>(grid, *a.tmap_k, *a.tmap_v, tkn, tvn, p, stream)
+                       : launch_tile_kernel<64, false, true>(grid, *a.tmap_k, *a.tmap_v, tkn, tvn, p, stream);
     else
-        e = a.d == 128 ? launch_tile_kernel<128, false>(grid, *a.tmap_k, *a.tmap_v, p, stream)
-                       : launch_tile_kernel<64, false>(grid, *a.tmap_k, *a.tmap_v, p, stream);
+        e = a.d == 128 ? launch_tile_kernel<128, false>(grid, *a.tmap_k, *a.tmap_v, tkn, tvn, p, stream)
+                       : launch_tile_kernel<64, false>(grid, *a.tmap_k, *a.tmap_v, tkn, tvn, p, stream);
     if (tr) tr->end(kKernelPrefill, stream);
     return e;
 }
@@ -686,8 +768,9 @@ cudaError_t launch_decode_prefix(const DecodeLayout &L, const DecodeArgs &a,
     // there measured much slower (l70b decode 345 -> 433 us per step).
     p.early_trigger = L.prefix_early;
     if (tr) tr->begin(kKernelDecodePrefix, stream);
-    cudaError_t e = L.d == 128 ? launch_tile_kernel<128, true>(grid, *a.tmap_k, *a.tmap_v, p, stream)
-                               : launch_tile_kernel<64, true>(grid, *a.tmap_k, *a.tmap_v, p, stream);
+    cudaError_t e = L.d == 128
+                        ? launch_tile_kernel<128, true>(grid, *a.tmap_k, *a.tmap_v, *a.tmap_k, *a.tmap_v, p, stream)
+                        : launch_tile_kernel<64, true>(grid, *a.tmap_k, *a.tmap_v, *a.tmap_k, *a.tmap_v, p, stream);
     if (tr) tr->end(kKernelDecodePrefix, stream);
     return e;
 }

@@ -44,7 +44,7 @@ EXPORTS = [
     "pkv_prefix_cache_evict", "pkv_prefix_cache_size", "pkv_prefix_groups_build",
     "pkv_selftest_wait_timeout", "pkv_lora_dispatch", "pkv_check_block_table",
     "paged_attn_verify_tree", "pkv_tree_masks", "pkv_blocks_staging_size", "pkv_blocks_gather",
-    "pkv_blocks_scatter", "pkv_lora_sgmv",
+    "pkv_blocks_scatter", "pkv_lora_sgmv", "paged_attn_prefill_append",
 ]
 
 
@@ -135,6 +135,7 @@ def load(path: str | None = None):
         "paged_attn_verify_tree": [V, V, V, V, V, V, V, i32, i32, i32, i32, f32, V, V],
         "pkv_tree_masks": [P, P, i32, P],
         "pkv_blocks_staging_size": [V, i32, ctypes.POINTER(sz)],
+        "paged_attn_prefill_append": [V, V, V, V, i32, V, V, V, V, V, i32, i32, i32, i32, f32, V],
         "pkv_lora_sgmv": [V, V, V, V, P, P, P, i32, i32, i32, i32, i32, i32, V, V, V],
         "pkv_blocks_gather": [V, V, i32, V, V],
         "pkv_blocks_scatter": [V, V, i32, V, V],
@@ -364,6 +365,32 @@ def paged_attn_prefill(pool, q, out, lse, cu_seqlens_q, context_lens, block_tabl
     _check(load().paged_attn_prefill(
         pool, _dptr(q), _dptr(out), _dptr(lse), _dptr(cu_seqlens_q), _dptr(context_lens),
         _dptr(block_table), int(block_table.shape[1]), int(context_lens.shape[0]),
+        int(max_seqlen_q), int(q.shape[1]), float(scale), _stream(stream)))
+
+
+def paged_attn_prefill_append(pool, q, k_new, v_new, out, lse, cu_seqlens_q, context_lens, block_table,
+                              max_seqlen_q: int, scale: float, stream=None):
+    """paged_attn_prefill with the new tokens' K/V (bf16 [T][Hkv][d], rows in
+    q's order) stored into the pool by the prefill kernel."""
+    import torch
+    _check_attn_args(pool, q, out, lse, context_lens, block_table, 0)
+    _need(tuple(out.shape) == tuple(q.shape), lambda: f"out must have q's shape {list(q.shape)}")
+    if lse is not None:
+        _need(lse.shape[0] == q.shape[0], lambda: f"lse must have {q.shape[0]} rows")
+    _check_tensor("cu_seqlens_q", cu_seqlens_q, torch.int32, 1)
+    _need(cu_seqlens_q.shape[0] == context_lens.shape[0] + 1,
+          lambda: f"cu_seqlens_q must have {context_lens.shape[0] + 1} entries")
+    T = int(q.shape[0])
+    geo = _pool_geometry(pool)
+    for name, t in (("k_new", k_new), ("v_new", v_new)):
+        ts = _check_tensor(name, t, torch.bfloat16, 3)
+        _need(ts[0] == T, lambda: f"{name} must have q's {T} rows, got {ts[0]}")
+        if geo is not None:
+            _need(ts[1] == geo[1] and ts[2] == geo[2],
+                  lambda: f"{name} rows must be [{geo[1]}][{geo[2]}], got {list(ts[1:])}")
+    _check(load().paged_attn_prefill_append(
+        pool, _dptr(q), _dptr(k_new), _dptr(v_new), T, _dptr(out), _dptr(lse), _dptr(cu_seqlens_q),
+        _dptr(context_lens), _dptr(block_table), int(block_table.shape[1]), int(context_lens.shape[0]),
         int(max_seqlen_q), int(q.shape[1]), float(scale), _stream(stream)))
 
 

@@ -36,6 +36,27 @@ def run_prefill(b, with_lse=True):
     return out, lse
 
 
+def run_prefill_append(b, with_lse=True):
+    """The prefill subset's write and attention in one call; the decode
+    subset's new tokens (if any) by kv_cache_write, so the pool ends as after
+    run_prefill."""
+    w = b.w
+    rows = B.new_token_rows(w, b.pre)
+    rows_d = B.new_token_rows(w, b.dec)
+    if rows_d.stop > rows_d.start:
+        pkv.kv_cache_write(b.pool, b.k_new[rows_d], b.v_new[rows_d], b.slots[rows_d])
+    n = rows.stop - rows.start
+    out = torch.full((n, w.num_q_heads, w.head_dim), float("nan"), dtype=torch.bfloat16, device="cuda")
+    lse = torch.full((n, w.num_q_heads), float("nan"), dtype=torch.float32, device="cuda") if with_lse else None
+    B.run_prefill_append(b, out, lse)
+    assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
+    return out, lse
+
+
+def _bits(t):
+    return t.view(torch.int16)
+
+
 def compare(b, out, lse, reqs, rows_per_req=None, threads=16, seed=0):
     """Compare every (or a sample of) query rows of the given requests."""
     w = b.w
@@ -111,7 +132,7 @@ def test_prefill_full_size_every_row(name):
     need_gpu()
     w = make_workload(name)
     b = B.build_batch(w, poison=True)
-    out, lse = run_prefill(b)
+    out, lse = run_prefill_append(b)   # the benchmark's call: write fused into the prefill
     assert torch.isfinite(out.float()).all() and torch.isfinite(lse).all()
     reqs = list(range(b.pre.start, b.pre.stop))
     pick = {reqs[0], reqs[-1], reqs[len(reqs) // 2], reqs[int(np.argmax(w.cached_lens[b.pre]))]}
@@ -119,6 +140,43 @@ def test_prefill_full_size_every_row(name):
     while len(pick) < min(8, len(reqs)):
         pick.add(int(rng.choice(reqs)))
     compare(b, out, lse, sorted(pick))
+    b.close()
+
+
+@pytest.mark.parametrize("name,scale", [("tiny", 1.0), ("l8b_prefill", 0.125), ("qwen_mixed", 0.125)])
+def test_prefill_append_equals_write_then_prefill(name, scale):
+    """paged_attn_prefill_append reads the new keys from k_new / v_new and
+    stores them from inside the prefill kernel: its outputs and LSE have the
+    bits of kv_cache_write + paged_attn_prefill, and the whole pool afterwards
+    (NaN-poisoned unused slots included) is bit-identical to theirs."""
+    need_gpu()
+    w = make_workload(name, scale_requests=scale)
+    b1 = B.build_batch(w, poison=True)
+    o1, l1 = run_prefill(b1)
+    k1, v1 = b1.k_cache.clone(), b1.v_cache.clone()
+    b1.close()
+    b2 = B.build_batch(w, poison=True)
+    o2, l2 = run_prefill_append(b2)
+    assert torch.equal(o1, o2) and torch.equal(l1, l2)
+    assert torch.equal(_bits(k1), _bits(b2.k_cache)) and torch.equal(_bits(v1), _bits(b2.v_cache))
+    compare(b2, o2, l2, range(b2.pre.start, b2.pre.stop), rows_per_req=16)
+    b2.close()
+
+
+def test_prefill_append_needs_block_aligned_cache():
+    """A request whose cached part is not whole blocks is skipped (output
+    untouched) and latches DEVICE_BOUNDS; the aligned one beside it is
+    computed and stored."""
+    need_gpu()
+    w = make_workload("custom", seed=41, custom=dict(Hq=8, Hkv=2, d=128, prefix_lens=[], group=[-1, -1],
+                                                   cached=[64, 100], new=[40, 30], decode=[False, False]))
+    b = B.build_batch(w, poison=True)
+    n = w.num_new_tokens
+    out = torch.full((n, 8, 128), float("nan"), dtype=torch.bfloat16, device="cuda")
+    B.run_prefill_append(b, out, None)
+    assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_ERR_DEVICE_BOUNDS
+    assert bool(torch.isnan(out[40:].float()).all())
+    compare(b, out, None, [0])
     b.close()
 
 
