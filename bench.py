@@ -340,10 +340,11 @@ def measure_workload(name, steps, warmup, use_groups=True, e2e_steps=0):
         # runs it: one paged_attn_decode_step call per step copies the step's
         # packed inputs (q, new K/V, context lengths) to the device, decodes
         # with the new tokens stored by the decode kernels
-        # (PKV_STEP_FUSED_WRITE) and copies the output back to pinned memory.  Alternate steps go to two streams, each with its own
-        # device input and output buffers; a step's kernels wait for the
-        # previous step's (one decode per pool at a time), so its copies
-        # overlap the other stream's kernels.  A pinned buffer is refilled
+        # (PKV_STEP_FUSED_WRITE) and copies the output back to pinned memory.
+        # Alternate steps go to two streams, each with its own device input
+        # and output buffers; a step's kernels wait for the previous step's
+        # (the steps share one workspace), so its copies overlap the other
+        # stream's kernels.  A pinned buffer is refilled
         # only after the step that last used it has completed.
         layout, host, _ = B.step_buffers(b, copies=2, fused=True)
         dev = [torch.empty(layout.bytes, dtype=torch.uint8, device=b.device) for _ in range(2)]

@@ -13,19 +13,23 @@
  * mapping (kv_slot_mapping), the prefix-caching index (pkv_prefix_cache_*)
  * and the prefix groups of a decode batch (pkv_prefix_groups_build),
  * the adapter-first, length-bucketed dispatch of a multi-adapter request
- * (pkv_lora_dispatch),
- * the cache write (kv_cache_write), suffix prefill (paged_attn_prefill),
- * decode (paged_attn_decode; without a caller workspace:
+ * (pkv_lora_dispatch) and the segmented multi-adapter LoRA projection
+ * (pkv_lora_sgmv), the cache write (kv_cache_write), suffix prefill
+ * (paged_attn_prefill; with the write fused in: paged_attn_prefill_append;
+ * tree-shaped draft verification: paged_attn_verify_tree, pkv_tree_masks),
+ * decode (paged_attn_decode; with the write fused in:
+ * paged_attn_decode_append; without a caller workspace:
  * paged_attn_decode_noalloc; one host-driven step with its copies:
- * paged_attn_decode_step), per-kernel tracing (pkv_trace_*), device error
- * reporting (pkv_check_device_errors) and a test aid for it
- * (pkv_selftest_wait_timeout).
+ * paged_attn_decode_step), KV-block transfer between pools
+ * (pkv_blocks_gather / pkv_blocks_scatter), per-kernel tracing
+ * (pkv_trace_*), device error reporting (pkv_check_device_errors), the host
+ * check of block tables (pkv_check_block_table) and a test aid for the
+ * bounded waits (pkv_selftest_wait_timeout).
  *
  * Conventions for every call
  *  - All device buffers are owned by the caller.  The library keeps host
- *    metadata (free list, reference counts, TMA descriptors) and 16 bytes of
- *    device words per pool (an error word and two work counters of the
- *    decode split pass), allocated by kv_pool_create.
+ *    metadata (free list, reference counts, TMA descriptors) and one 4-byte
+ *    device word per pool (its error word), allocated by kv_pool_create.
  *  - "device" pointers are CUDA global-memory addresses on the pool's device;
  *    "host" pointers are ordinary CPU memory.  Device buffers must be 16-byte
  *    aligned and contiguous in the stated layout.
@@ -40,10 +44,11 @@
  *  - Element type: bf16 only.  Block size: 16 tokens.  Head dim: 64 or 128.
  *    num_q_heads must be a multiple of num_kv_heads; q heads h belong to kv
  *    head h / (num_q_heads / num_kv_heads) (contiguous GQA grouping).
- *  - A pool handle is not thread-safe; calls on one handle must not overlap.
- *    In particular at most one decode per pool may be in flight on the GPU
- *    at a time (its split pass takes work from the pool's counters): decodes
- *    on several streams need one pool each, or an event between them.
+ *  - A pool handle is not thread-safe; calls on one handle must not overlap
+ *    in time on the host.  On the GPU the kernels of one pool share only its
+ *    error word, so launches on several streams may be in flight together as
+ *    long as each has its own workspace and outputs and they write no common
+ *    slots.  Different pools may be used from different host threads.
  */
 #ifndef PKV_H
 #define PKV_H
@@ -471,8 +476,8 @@ typedef struct pkv_step_layout {
  * before the output copy.  With two streams taking alternate steps, each
  * with its own dev_in, out and lse, and each step waiting for the previous
  * step's done_event, a step's copies overlap the other stream's kernels
- * while the kernels themselves stay in order (at most one decode per pool in
- * flight).
+ * while the kernels themselves stay in order (so the steps may share one
+ * workspace).
  * The caller keeps host_in, host_out and host_lse untouched until the stream
  * has passed the step (an event recorded after the call).  Other arguments
  * and the errors are those of kv_cache_write and paged_attn_decode;
