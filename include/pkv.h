@@ -16,7 +16,9 @@
  * (pkv_lora_dispatch) and the segmented multi-adapter LoRA projection
  * (pkv_lora_sgmv), the cache write (kv_cache_write), suffix prefill
  * (paged_attn_prefill; with the write fused in: paged_attn_prefill_append;
- * tree-shaped draft verification: paged_attn_verify_tree, pkv_tree_masks),
+ * tree-shaped draft verification: paged_attn_verify_tree, pkv_tree_masks;
+ * with each group's shared prefix read once: paged_attn_verify_tree_grouped,
+ * pkv_verify_groups_build),
  * decode (paged_attn_decode; with the write fused in:
  * paged_attn_decode_append; without a caller workspace:
  * paged_attn_decode_noalloc; one host-driven step with its copies:
@@ -381,6 +383,68 @@ int paged_attn_verify_tree(pkv_pool_t pool, const void *q, void *out, float *lse
                            const int32_t *block_table, int32_t max_blocks, int32_t num_requests,
                            int32_t max_seqlen_q, int32_t num_q_heads, float scale,
                            const uint64_t *tree_mask, pkv_stream_t stream);
+
+/* Shared-prefix groups of a verification batch (Sec. 5.3 with Sec. 5.4):
+ * the draft tokens of the requests that share a cached prefix, grouped so
+ * that the prefix is read once per group and kv head rather than once per
+ * request.  Group g's requests all name the same group_blocks[g] physical
+ * blocks first in their table rows (full blocks of the shared prefix, before
+ * every draft); member_token lists the draft tokens (rows of q) of those
+ * requests.  All arrays are device arrays; pkv_verify_groups_build makes them
+ * (on the host) from each request's group.  As with pkv_prefix_groups, the
+ * host bounds size the workspace and the grid and are not checked against
+ * the device arrays: members or blocks past a bound are left out. */
+typedef struct {
+    int32_t num_groups;        /* G >= 0; 0: no sharing, every key in the private pass */
+    int32_t max_group_blocks;  /* host upper bound on group_blocks[g]             */
+    int32_t max_group_tokens;  /* host upper bound on the draft tokens of a group */
+    int32_t reserved;          /* 0                                               */
+    const int32_t *group_start;   /* [G+1] CSR offsets into member_token          */
+    const int32_t *member_token;  /* [group_start[G]] draft-token rows, by group  */
+    const int32_t *group_blocks;  /* [G] shared leading blocks of group g         */
+    const int32_t *group_row;     /* [G] a block-table row (request) of group g   */
+    const int32_t *request_group; /* [num_requests] group of request r, -1: none  */
+} pkv_verify_groups;
+
+/* Bytes of workspace paged_attn_verify_tree_grouped needs (host call).
+ * num_tokens: draft tokens of the batch (cu_seqlens_q[num_requests]); groups
+ * may be NULL.  Errors: INVALID_ARG. */
+int paged_attn_verify_tree_workspace_size(pkv_pool_t pool, int32_t num_tokens, int32_t num_q_heads,
+                                          int32_t max_blocks, const pkv_verify_groups *groups,
+                                          size_t *bytes_out);
+
+/* paged_attn_verify_tree with the shared prefix of each group read once per
+ * group and kv head: a tensor-core pass over each group's draft tokens and
+ * its shared blocks (all visible to every draft), a pass over each request's
+ * keys after them (its private context and its drafts, under the draft
+ * masks), and the log-sum-exp merge of the two.  Same result as
+ * paged_attn_verify_tree up to rounding (the merge of two partial softmaxes).
+ *  num_tokens: cu_seqlens_q[num_requests] (host).  groups: as above, or NULL.
+ *  A grouped request's cached part, context_lens[r] - n_r, must cover its
+ *  group's blocks (else it latches DEVICE_BOUNDS and its outputs are
+ *  undefined).
+ *  workspace: device, 256-byte aligned, at least
+ *  paged_attn_verify_tree_workspace_size() bytes; holds partials between the
+ *  passes.
+ * Errors: those of paged_attn_verify_tree; UNSUPPORTED beyond 8 q heads per kv
+ * head; WORKSPACE. */
+int paged_attn_verify_tree_grouped(pkv_pool_t pool, const void *q, void *out, float *lse,
+                                   const int32_t *cu_seqlens_q, const int32_t *context_lens,
+                                   const int32_t *block_table, int32_t max_blocks, int32_t num_requests,
+                                   int32_t num_tokens, int32_t max_seqlen_q, int32_t num_q_heads, float scale,
+                                   const uint64_t *tree_mask, const pkv_verify_groups *groups,
+                                   void *workspace, size_t workspace_bytes, pkv_stream_t stream);
+
+/* Token groups of a verification batch (host): from cu_seqlens ([R+1],
+ * cu_seqlens[0] = 0) and request_group ([R], values in [-1, num_groups)),
+ * writes group_start_out [num_groups + 1], member_token_out
+ * [cu_seqlens[R]] (the draft tokens of group 0's requests in request order,
+ * then group 1's, ...; tokens of ungrouped requests are not listed),
+ * group_row_out [num_groups] (the group's first request, -1 if it has none)
+ * and *max_group_tokens_out.  All host arrays.  Errors: INVALID_ARG. */
+int pkv_verify_groups_build(const int32_t *cu_seqlens, const int32_t *request_group, int32_t num_requests,
+                            int32_t num_groups, int32_t *group_start_out, int32_t *member_token_out,
+                            int32_t *group_row_out, int32_t *max_group_tokens_out);
 
 /* Draft masks of tree-shaped drafts (host): parent[cu_seqlens[r] + i] is the
  * draft that draft i of request r continues (-1: the context), an earlier

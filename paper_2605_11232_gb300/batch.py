@@ -253,6 +253,41 @@ def run_prefill_append(b: Batch, out: torch.Tensor, lse, stream=None):
                                   b.context_lens[b.pre], b.table[b.pre], b.max_seqlen_pre, b.w.scale, stream)
 
 
+def verify_groups(b: Batch):
+    """Token groups of the prefill subset's requests for grouped verification:
+    (pkv.VerifyGroups, the device tensors it points to; keep them alive)."""
+    w = b.w
+    req = range(b.pre.start, b.pre.stop)
+    G = len(w.prefix_lens)
+    rg = np.array([int(w.group_of_req[r]) for r in req], np.int32)
+    cu = np.zeros(len(rg) + 1, np.int32)
+    cu[1:] = np.cumsum(w.new_lens[b.pre])
+    tg = pkv.pkv_verify_groups_build(cu, rg, G)
+    gblocks = np.array([P // 16 for P in w.prefix_lens], np.int32)
+    dev = dict(group_start=torch.from_numpy(tg["group_start"]).to(b.device),
+               member_token=torch.from_numpy(tg["member_token"]).to(b.device),
+               group_blocks=torch.from_numpy(gblocks).to(b.device),
+               group_row=torch.from_numpy(tg["group_row"]).to(b.device),
+               request_group=torch.from_numpy(rg).to(b.device))
+    vg = pkv.make_verify_groups(G, int(gblocks.max()) if G else 0, tg["max_group_tokens"], **dev)
+    return vg, dev
+
+
+def verify_workspace(b: Batch, groups) -> torch.Tensor:
+    rows = new_token_rows(b.w, b.pre)
+    nbytes = pkv.paged_attn_verify_tree_workspace_size(b.pool, rows.stop - rows.start, b.w.num_q_heads,
+                                                       b.table.shape[1], groups)
+    return torch.empty(max(nbytes, 256), dtype=torch.uint8, device=b.device)
+
+
+def run_verify_grouped(b: Batch, out: torch.Tensor, lse, tree_mask: torch.Tensor, groups, ws: torch.Tensor,
+                       max_seqlen_q: int | None = None, stream=None):
+    rows = new_token_rows(b.w, b.pre)
+    pkv.paged_attn_verify_tree_grouped(b.pool, b.q[rows], out, lse, b.cu_pre, b.context_lens[b.pre],
+                                       b.table[b.pre], max_seqlen_q or b.max_seqlen_pre, b.w.scale, tree_mask,
+                                       groups, ws, stream)
+
+
 def kv_waste(b: Batch) -> float:
     """Fraction of allocated KV slots holding no token, shared blocks once."""
     used_blocks = b.num_blocks_pool - pkv.kv_pool_num_free(b.pool)

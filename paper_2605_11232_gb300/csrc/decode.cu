@@ -261,15 +261,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     constexpr uint32_t kTileBytes = kHalves * 2048;   // one K or V tile of a (block, kv head)
     constexpr uint32_t kSlotBytes = 2 * kTileBytes;
     constexpr int CPR = D / 8;                        // 16-byte chunks per key row
-    constexpr uint32_t kQBytes = 8 * D * 2;           // Q area of a stage: 8 head rows
+    const uint32_t kQBytes = (uint32_t)lay.qbytes;    // Q area of a stage: 4 or 8 head rows
     const int S = lay.stages;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                 ~uintptr_t(1023));
-    // K/V stages [kWarps][S] | Q areas [kWarps][S] | descriptors [kWarps][S] |
-    // full barriers [kWarps][S] | plan [R + 1] | context lengths [R] (if they fit)
+    // K/V stages [kWarps][S] | Q areas [kWarps][S] | slack | descriptors
+    // [kWarps][S] | full barriers [kWarps][S] | plan [R + 1] | context lengths
+    // [R] (if they fit).  The Q fragments are read as 8 head rows; with 4-row
+    // areas (g <= 4) rows 4-7 come from the next area, or from the slack after
+    // the last one, and feed only head columns that are never written out.
     const uint32_t qbase = smem_u32(smem) + (uint32_t)(kWarps * S) * kSlotBytes;
-    SlotDesc *descs = reinterpret_cast<SlotDesc *>(smem + (size_t)kWarps * S * (kSlotBytes + kQBytes));
+    SlotDesc *descs = reinterpret_cast<SlotDesc *>(smem + (size_t)kWarps * S * (kSlotBytes + kQBytes) +
+                                                   (8 * D * 2 - kQBytes));
     uint64_t *bars = reinterpret_cast<uint64_t *>(descs + kWarps * S);
     int32_t *P = reinterpret_cast<int32_t *>(bars + kWarps * S);
     int32_t *Ls = lay.lens_in_smem ? P + lay.R + 1 : nullptr;
@@ -680,10 +684,26 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(DecodeArgs a, Decod
 namespace {
 
 // Shared memory of the split pass for `stages` ring stages.
-size_t split_smem_bytes(int32_t R, int32_t d, int stages, bool lens) {
-    const size_t slot = 2 * (size_t)(d / 64) * 2048 + 8 * (size_t)d * 2;   // K/V tiles + Q area
-    return 1024 + (size_t)kWarps * stages * (slot + sizeof(SlotDesc) + 8) + 4 * ((size_t)R + 1) +
-           (lens ? 4 * (size_t)R : 0);
+// qbytes: the Q area of a stage (4 or 8 head rows of d bf16)
+size_t split_smem_bytes(int32_t R, int32_t d, int stages, bool lens, size_t qbytes) {
+    const size_t slot = 2 * (size_t)(d / 64) * 2048 + qbytes;   // K/V tiles + Q area
+    return 1024 + (size_t)kWarps * stages * (slot + sizeof(SlotDesc) + 8) + (8 * (size_t)d * 2 - qbytes) +
+           4 * ((size_t)R + 1) + (lens ? 4 * (size_t)R : 0);
+}
+
+}  // namespace
+
+namespace {
+
+// Workspace offsets for prefix_parts + private_parts part slots per (row, q head).
+void set_part_slots(DecodeLayout &L, int private_parts) {
+    L.parts_per_head = L.prefix_parts + private_parts;
+    const size_t slots = (size_t)L.R * L.Hq * L.parts_per_head;
+    auto up = [](size_t x) { return (x + 255) & ~(size_t)255; };
+    L.off_o = 0;
+    L.off_ml = up(slots * L.d * sizeof(float));
+    L.off_nparts = L.off_ml + up(slots * sizeof(float2));
+    L.total = L.off_nparts + up((size_t)L.R * L.Hkv * sizeof(int32_t));
 }
 
 }  // namespace
@@ -742,20 +762,28 @@ DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_
     }
     L.split_grid = L.prefix_early ? sms - (int32_t)L.prefix_ctas : sms;
     // as many ring stages as fit (the plan takes 4 bytes per request)
+    // as many ring stages as fit: each warp keeps S - 1 blocks in flight while
+    // it computes on one, and 2 stages leave the pass short of HBM on ~120 SMs
+    L.qbytes = (L.g <= 4 ? 4 : 8) * d * 2;
     L.stages = 2;
     const int max_stages = d == 64 ? 4 : 3;
     for (int st = max_stages; st > 2; --st)
-        if (split_smem_bytes(R, d, st, false) <= kMaxSmemPerBlock) { L.stages = st; break; }
+        if (split_smem_bytes(R, d, st, false, L.qbytes) <= kMaxSmemPerBlock) { L.stages = st; break; }
     // the context lengths beside the plan when they fit (saves a global read per piece list)
-    L.lens_in_smem = split_smem_bytes(R, d, L.stages, true) <= kMaxSmemPerBlock ? 1 : 0;
-    L.split_smem = split_smem_bytes(R, d, L.stages, L.lens_in_smem != 0);
-    L.parts_per_head = L.prefix_parts + kMaxPrivateParts;
-    const size_t slots = (size_t)R * Hq * L.parts_per_head;
-    auto up = [](size_t x) { return (x + 255) & ~(size_t)255; };
-    L.off_o = 0;
-    L.off_ml = up(slots * d * sizeof(float));
-    L.off_nparts = L.off_ml + up(slots * sizeof(float2));
-    L.total = L.off_nparts + up((size_t)R * Hkv * sizeof(int32_t));
+    L.lens_in_smem = split_smem_bytes(R, d, L.stages, true, L.qbytes) <= kMaxSmemPerBlock ? 1 : 0;
+    L.split_smem = split_smem_bytes(R, d, L.stages, L.lens_in_smem != 0, L.qbytes);
+    set_part_slots(L, kMaxPrivateParts);
+    return L;
+}
+
+DecodeLayout verify_layout(int32_t T, int32_t Hq, int32_t Hkv, int32_t d, int32_t max_blocks,
+                           int32_t num_groups, int32_t max_group_blocks, int32_t max_group_tokens,
+                           int32_t num_sms) {
+    // the prefix pass of decode over draft tokens, and one private part per
+    // token (the tile pass over the request's keys after the shared blocks)
+    DecodeLayout L = decode_layout(T, Hq, Hkv, d, max_blocks, num_groups, max_group_blocks, max_group_tokens,
+                                   num_sms);
+    set_part_slots(L, 1);
     return L;
 }
 
@@ -780,15 +808,25 @@ static cudaError_t launch_decode_t(const DecodeLayout &L, const DecodeArgs &a, i
                                *a.tmap_k, *a.tmap_v, a, L, num_blocks_pool, prefix ? 1 : 0);
     if (tr) tr->end(kKernelDecodeSplit, stream);
     if (e != cudaSuccess) return e;
+    return launch_decode_combine(L, a, stream, tr);
+}
+
+template <int D>
+static cudaError_t launch_combine_t(const DecodeLayout &L, const DecodeArgs &a, cudaStream_t stream, Tracer *tr) {
     // four warps per CTA: small batches spread over more SMs
     const int64_t items = (int64_t)L.R * L.Hkv;
     const int64_t cgrid = (items + 3) / 4;
     if (cgrid > 0x7fffffff) return cudaErrorInvalidConfiguration;
     if (tr) tr->begin(kKernelDecodeCombine, stream);
-    e = L.g <= 4 ? launch_pdl(decode_combine_kernel<D, 4>, dim3((unsigned)cgrid), dim3(128), 0, stream, a, L)
-                 : launch_pdl(decode_combine_kernel<D, 8>, dim3((unsigned)cgrid), dim3(128), 0, stream, a, L);
+    cudaError_t e = L.g <= 4
+                        ? launch_pdl(decode_combine_kernel<D, 4>, dim3((unsigned)cgrid), dim3(128), 0, stream, a, L)
+                        : launch_pdl(decode_combine_kernel<D, 8>, dim3((unsigned)cgrid), dim3(128), 0, stream, a, L);
     if (tr) tr->end(kKernelDecodeCombine, stream);
     return e;
+}
+
+cudaError_t launch_decode_combine(const DecodeLayout &L, const DecodeArgs &a, cudaStream_t stream, Tracer *tr) {
+    return L.d == 128 ? launch_combine_t<128>(L, a, stream, tr) : launch_combine_t<64>(L, a, stream, tr);
 }
 
 cudaError_t launch_decode(const DecodeLayout &L, const DecodeArgs &a, int32_t num_blocks_pool,

@@ -546,6 +546,136 @@ int paged_attn_verify_tree(pkv_pool_t pool, const void *q, void *out, float *lse
                         num_requests, max_seqlen_q, num_q_heads, scale, tree_mask, nullptr, nullptr, 0, stream);
 }
 
+int paged_attn_verify_tree_workspace_size(pkv_pool_t pool, int32_t num_tokens, int32_t num_q_heads,
+                                          int32_t max_blocks, const pkv_verify_groups *groups,
+                                          size_t *bytes_out) {
+    if (!pool || !bytes_out || num_tokens < 0 || num_q_heads <= 0 || max_blocks <= 0)
+        return fail(PKV_ERR_INVALID_ARG, "bad arguments");
+    const bool grouped = groups && groups->num_groups > 0;
+    pkv::DecodeLayout L = pkv::verify_layout(num_tokens, num_q_heads, pool->desc.num_kv_heads,
+                                             pool->desc.head_dim, max_blocks, grouped ? groups->num_groups : 0,
+                                             grouped ? groups->max_group_blocks : 0,
+                                             grouped ? groups->max_group_tokens : 0, pool->num_sms);
+    *bytes_out = L.total;
+    return ok();
+}
+
+int paged_attn_verify_tree_grouped(pkv_pool_t pool, const void *q, void *out, float *lse,
+                                   const int32_t *cu_seqlens_q, const int32_t *context_lens,
+                                   const int32_t *block_table, int32_t max_blocks, int32_t num_requests,
+                                   int32_t num_tokens, int32_t max_seqlen_q, int32_t num_q_heads, float scale,
+                                   const uint64_t *tree_mask, const pkv_verify_groups *groups,
+                                   void *workspace, size_t workspace_bytes, pkv_stream_t stream) {
+    int rc = check_kernel_pool(pool);
+    if (rc != PKV_OK) return rc;
+    const pkv_pool_desc &d = pool->desc;
+    if (num_requests < 0 || num_tokens < 0 || max_seqlen_q < 0 || max_blocks <= 0)
+        return fail(PKV_ERR_INVALID_ARG, "bad sizes");
+    if (num_q_heads <= 0 || num_q_heads % d.num_kv_heads != 0)
+        return fail(PKV_ERR_INVALID_ARG, "num_q_heads must be a positive multiple of num_kv_heads");
+    if (num_q_heads / d.num_kv_heads > 8)
+        return fail(PKV_ERR_UNSUPPORTED, "grouped verification supports up to 8 q heads per kv head");
+    if (max_seqlen_q > 64) return fail(PKV_ERR_UNSUPPORTED, "at most 64 draft tokens per request");
+    if (max_blocks > pkv::kPrefillMaxBlocks)
+        return fail(PKV_ERR_UNSUPPORTED, "table width %d: verification supports up to %d blocks", max_blocks,
+                    pkv::kPrefillMaxBlocks);
+    if (num_tokens > (1 << 20)) return fail(PKV_ERR_UNSUPPORTED, "more than 2^20 draft tokens");
+    if (!(scale > 0.f) || !std::isfinite(scale)) return fail(PKV_ERR_INVALID_ARG, "bad scale");
+    if (num_requests == 0 || max_seqlen_q == 0 || num_tokens == 0) return ok();
+    if (!q || !out || !cu_seqlens_q || !context_lens || !block_table)
+        return fail(PKV_ERR_INVALID_ARG, "NULL buffer");
+    if (!aligned16(q) || !aligned16(out)) return fail(PKV_ERR_INVALID_ARG, "misaligned q/out");
+    if (!tree_mask || (reinterpret_cast<uintptr_t>(tree_mask) & 7))
+        return fail(PKV_ERR_INVALID_ARG, "tree_mask must be a non-NULL, 8-byte aligned device array");
+    int32_t G = 0, mgb = 0, mgt = 0;
+    if (groups && groups->num_groups > 0) {
+        G = groups->num_groups;
+        mgb = groups->max_group_blocks;
+        mgt = groups->max_group_tokens;
+        if (!groups->group_start || !groups->member_token || !groups->group_blocks || !groups->group_row ||
+            !groups->request_group || mgb < 0 || mgt < 0)
+            return fail(PKV_ERR_INVALID_ARG, "incomplete verification-group descriptor");
+        if (mgb > max_blocks) return fail(PKV_ERR_INVALID_ARG, "max_group_blocks exceeds the table width");
+        if ((int64_t)G * d.num_kv_heads > INT32_MAX) return fail(PKV_ERR_UNSUPPORTED, "too many groups");
+    }
+    const pkv::DecodeLayout L = pkv::verify_layout(num_tokens, num_q_heads, d.num_kv_heads, d.head_dim,
+                                                   max_blocks, G, mgb, mgt, pool->num_sms);
+    if (!workspace || workspace_bytes < L.total)
+        return fail(PKV_ERR_WORKSPACE, "workspace of %zu bytes needed", L.total);
+    if (reinterpret_cast<uintptr_t>(workspace) & 255)
+        return fail(PKV_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+    if ((rc = set_device(pool)) != PKV_OK) return rc;
+    if ((rc = build_tmaps(pool)) != PKV_OK) return rc;
+    const float scale_log2 = scale * 1.4426950408889634f;
+    pkv::DecodeArgs a{};
+    a.q = q; a.out = out; a.lse = lse;
+    a.block_table = block_table; a.max_blocks = max_blocks;
+    a.scale_log2 = scale_log2;
+    a.num_groups = G;
+    if (G > 0) {
+        a.max_group_members = mgt;
+        a.group_start = groups->group_start; a.member_req = groups->member_token;
+        a.group_blocks = groups->group_blocks;
+        a.group_row = groups->group_row;
+        a.num_table_rows = num_requests;
+    }
+    a.ws = workspace;
+    a.err = pool->d_err;
+    a.tmap_k = &pool->tmap_k; a.tmap_v = &pool->tmap_v;
+    pkv::PrefillArgs pa{};
+    pa.q = q;
+    pa.cu_seqlens_q = cu_seqlens_q; pa.context_lens = context_lens;
+    pa.block_table = block_table; pa.max_blocks = max_blocks;
+    pa.R = num_requests; pa.Hq = num_q_heads; pa.Hkv = d.num_kv_heads; pa.d = d.head_dim;
+    pa.max_seqlen_q = max_seqlen_q;
+    pa.num_blocks_pool = d.num_blocks;
+    pa.scale_log2 = scale_log2;
+    pa.tmap_k = &pool->tmap_k; pa.tmap_v = &pool->tmap_v;
+    pa.err = pool->d_err;
+    pa.tree_mask = reinterpret_cast<const unsigned long long *>(tree_mask);
+    cudaError_t e = pkv::launch_verify_grouped(L, a, pa, G > 0 ? groups->request_group : nullptr,
+                                               static_cast<cudaStream_t>(stream), pool->tracer);
+    if (e != cudaSuccess) return cuda_fail(e, "paged_attn_verify_tree_grouped launch");
+    return ok();
+}
+
+int pkv_verify_groups_build(const int32_t *cu_seqlens, const int32_t *request_group, int32_t num_requests,
+                            int32_t num_groups, int32_t *group_start_out, int32_t *member_token_out,
+                            int32_t *group_row_out, int32_t *max_group_tokens_out) {
+    if (num_requests < 0 || num_groups < 0 || !cu_seqlens || !group_start_out || !max_group_tokens_out ||
+        (num_requests > 0 && !request_group) || (num_groups > 0 && !group_row_out))
+        return fail(PKV_ERR_INVALID_ARG, "bad arguments");
+    if (cu_seqlens[0] != 0) return fail(PKV_ERR_INVALID_ARG, "cu_seqlens[0] must be 0");
+    std::vector<int64_t> count(num_groups, 0);
+    for (int32_t r = 0; r < num_requests; ++r) {
+        const int32_t n = cu_seqlens[r + 1] - cu_seqlens[r];
+        if (n < 0) return fail(PKV_ERR_INVALID_ARG, "cu_seqlens decreases at request %d", r);
+        const int32_t gr = request_group[r];
+        if (gr < -1 || gr >= num_groups)
+            return fail(PKV_ERR_INVALID_ARG, "request %d: group %d out of range", r, gr);
+        if (gr >= 0) count[gr] += n;
+    }
+    if (num_requests > 0 && cu_seqlens[num_requests] > 0 && !member_token_out)
+        return fail(PKV_ERR_INVALID_ARG, "NULL member_token_out");
+    int64_t total = 0, mx = 0;
+    for (int32_t g = 0; g < num_groups; ++g) {
+        group_start_out[g] = (int32_t)total;
+        group_row_out[g] = -1;
+        total += count[g];
+        mx = std::max(mx, count[g]);
+    }
+    group_start_out[num_groups] = (int32_t)total;
+    std::vector<int64_t> fill(group_start_out, group_start_out + num_groups);
+    for (int32_t r = 0; r < num_requests; ++r) {
+        const int32_t gr = request_group[r];
+        if (gr < 0) continue;
+        if (group_row_out[gr] < 0) group_row_out[gr] = r;
+        for (int32_t t = cu_seqlens[r]; t < cu_seqlens[r + 1]; ++t) member_token_out[fill[gr]++] = t;
+    }
+    *max_group_tokens_out = (int32_t)mx;
+    return ok();
+}
+
 int pkv_tree_masks(const int32_t *parent, const int32_t *cu_seqlens, int32_t num_requests,
                    uint64_t *masks_out) {
     if (num_requests < 0 || !cu_seqlens || (num_requests > 0 && cu_seqlens[num_requests] > 0 &&

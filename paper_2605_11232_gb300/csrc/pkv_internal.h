@@ -108,6 +108,7 @@ struct DecodeLayout {
     int32_t prefix_early;        // the prefix pass lets the split pass start beside it
     int32_t split_grid;          // split-pass CTAs beside an early prefix pass
     int32_t stages;              // ring stages per warp of the split pass
+    int32_t qbytes;              // bytes of a stage's Q area (4 or 8 head rows)
     int32_t lens_in_smem;        // the split pass keeps the context lengths in shared memory
     size_t split_smem;           // dynamic shared memory of the split pass
     int32_t parts_per_head;      // prefix_parts + kMaxPrivateParts
@@ -120,6 +121,12 @@ struct DecodeLayout {
 
 DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_t max_blocks,
                            int32_t num_groups, int32_t max_group_blocks, int32_t max_group_members,
+                           int32_t num_sms);
+
+// Grouped verification: decode's layout with rows = draft tokens (T) and one
+// private part slot per (token, q head).
+DecodeLayout verify_layout(int32_t T, int32_t Hq, int32_t Hkv, int32_t d, int32_t max_blocks,
+                           int32_t num_groups, int32_t max_group_blocks, int32_t max_group_tokens,
                            int32_t num_sms);
 
 cudaError_t launch_cache_write(const void *k_new, const void *v_new, const int64_t *slots,
@@ -151,10 +158,20 @@ struct DecodeArgs {
     // by the split pass (paged_attn_decode_append); null: already in the cache
     const void *k_new;
     const void *v_new;
+    // grouped verification: the table row naming each group's prefix blocks
+    // (null: the first member's) and the number of table rows
+    const int32_t *group_row;
+    int32_t num_table_rows;
 };
 
 cudaError_t launch_decode(const DecodeLayout &L, const DecodeArgs &a, int32_t num_blocks_pool,
                           cudaStream_t stream, Tracer *tr);
+
+// The combine alone: merge every (row, kv head)'s partials of the workspace
+// into out / lse (rows = L.R; decode requests, or draft tokens).
+cudaError_t launch_decode_combine(const DecodeLayout &L, const DecodeArgs &a, cudaStream_t stream, Tracer *tr);
+
+
 
 // Bit copy of n blocks (device ids) between a pool's caches and a staging
 // buffer [n][K, V][Hkv][16][d] (transfer.cu).
@@ -186,6 +203,15 @@ struct PrefillArgs {
 };
 
 cudaError_t launch_prefill(const PrefillArgs &a, cudaStream_t stream, Tracer *tr);
+
+// Grouped verification of tree-shaped drafts: the shared-prefix pass over each
+// group's draft tokens, the private pass (keys after the shared blocks, draft
+// masks) writing partial slot L.prefix_parts, then the combine over the
+// tokens.  a: the decode arguments with rows = draft tokens (a.q, a.out,
+// a.lse over [T]; groups over tokens, a.group_row / a.num_table_rows set);
+// pa: the prefill arguments of the private pass (tree_mask set).
+cudaError_t launch_verify_grouped(const DecodeLayout &L, const DecodeArgs &a, const PrefillArgs &pa,
+                                  const int32_t *request_group, cudaStream_t stream, Tracer *tr);
 
 // Shared-prefix pass of decode (tcgen05 tile kernel in prefix mode): partials
 // of every group member over its group's prefix blocks, split in key ranges of

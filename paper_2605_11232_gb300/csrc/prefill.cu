@@ -107,6 +107,18 @@ struct KernelParams {
     int32_t fused;
     const uint16_t *k_new, *v_new;   // [T][Hkv][D]
     uint16_t *k_cache, *v_cache;     // the pool
+    // shared-prefix pass over draft tokens (grouped verification): the table
+    // row naming each group's prefix blocks (null: the first member's row,
+    // the member ids being requests) and the number of table rows
+    const int32_t *group_row;
+    int32_t num_table_rows;
+    // private pass of grouped verification (PART): each request's keys after
+    // its group's shared blocks, written as part slot private_part
+    const int32_t *request_group;    // [R] group of each request, -1: none
+    int32_t private_part;
+    int32_t prefix_parts;            // prefix part slots (their count per request goes to nparts)
+    int32_t *nparts;                 // [T * Hkv] part counts (private | prefix << 16)
+    int32_t after_prefix;            // a shared-prefix pass precedes (and started) this pass
 };
 
 // Row maximum of the 128 raw scores a thread holds (8 independent chains).
@@ -164,13 +176,18 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
 //   item, key split); tile X row i = member X*tpt + i / g of the item; keys =
 //   the split's range of the group's prefix blocks (read through the first
 //   member's table row), all visible; writes unnormalised partials.
-template <int D, bool PREFIX, bool TREE = false, bool FUSED = false>
+template <int D, bool PREFIX, bool TREE = false, bool FUSED = false, bool PART = false>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tile_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
                      const __grid_constant__ CUtensorMap tmkn, const __grid_constant__ CUtensorMap tmvn,
                      const KernelParams p) {
     using Ly = Layout<D>;
-    pdl_wait();
+    // The private pass of grouped verification runs beside the shared-prefix
+    // pass, which started it after its own wait: nothing read here is written
+    // by that pass, so it waits for it only before leaving (the combine needs
+    // both).  Every other mode, and a private pass with no prefix pass before
+    // it, waits for the preceding kernel first.
+    if (!PART || !p.after_prefix) pdl_wait();
     if constexpr (PREFIX) {
         if (p.early_trigger) pdl_trigger();   // the split pass may start on the free SMs
     }
@@ -184,11 +201,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         cu0 = __ldg(p.cu_seqlens_q + r);
         const int n_r = __ldg(p.cu_seqlens_q + r + 1) - cu0;
         q0 = item * 2 * p.tpt;
-        if (q0 >= n_r) return;
+        if (q0 >= n_r) {
+            if constexpr (PART) pdl_wait();
+            return;
+        }
         nq = min(2 * p.tpt, n_r - q0);
         const int L = __ldg(p.context_lens + r);
         if (L < n_r || L > 16 * p.max_blocks) {
             if (threadIdx.x == 0) latch_error(p.err, kDevBounds);
+            if constexpr (PART) pdl_wait();
             return;
         }
         cached = L - n_r;                 // keys before the request's new tokens
@@ -202,6 +223,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         q_pos0 = L - n_r + q0;            // absolute position of the item's first query
         kv_end = q_pos0 + nq;             // keys [0, kv_end) are visible to some row
+        if constexpr (PART) {
+            // keys from the end of the group's shared blocks; positions from
+            // here on count from there
+            const int grp = p.request_group ? __ldg(p.request_group + r) : -1;
+            blk_off = grp >= 0 ? __ldg(p.group_blocks + grp) : 0;
+            if (blk_off < 0 || blk_off * 16 > q_pos0) {
+                if (threadIdx.x == 0) latch_error(p.err, kDevBounds);
+                pdl_wait();
+                return;
+            }
+            q_pos0 -= blk_off * 16;
+            kv_end -= blk_off * 16;
+        }
         nblk = (kv_end + 15) >> 4;
         trow = p.block_table + (int64_t)r * p.max_blocks;
     } else {
@@ -221,11 +255,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         kv_end = nblk * 16;
         nq = min(2 * p.tpt, nm - mt0);
         m0 = gs + mt0;
-        // every member id of this item (and the first member, whose table row
-        // names the prefix blocks) must be a request of the batch: thread i
-        // checks member i (nq <= 256 < kThreads)
-        const int r_first = __ldg(p.member_req + gs);
-        bool bad = r_first < 0 || r_first >= p.num_requests;
+        // every member id of this item must be below num_requests, and the
+        // table row naming the prefix blocks (the first member's, or the
+        // group's own) a row of the table: thread i checks member i
+        // (nq <= 256 < kThreads)
+        const int r_first = p.group_row ? __ldg(p.group_row + grp) : __ldg(p.member_req + gs);
+        bool bad = r_first < 0 || r_first >= (p.group_row ? p.num_table_rows : p.num_requests);
         if (threadIdx.x < nq) {
             const int rm = __ldg(p.member_req + m0 + threadIdx.x);
             bad = bad || rm < 0 || rm >= p.num_requests;
@@ -238,6 +273,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (nblk > kMaxItemBlocks) {
         if (threadIdx.x == 0) latch_error(p.err, kDevBounds);
+        if constexpr (PART) pdl_wait();
         return;
     }
     const int nkt = (kv_end + kKeys - 1) / kKeys;
@@ -629,7 +665,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 __syncwarp();
             };
-            if constexpr (!PREFIX) {
+            if constexpr (!PREFIX && !PART) {
                 const float inv = 1.0f / l;
                 // bf16 rows of D values: D * 2 bytes <= RB
 #pragma unroll
@@ -652,8 +688,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 });
                 if (valid && p.lse) p.lse[row_idx[x * kRows + row]] = (m + __log2f(l)) * 0.69314718055994530942f;
             } else {
-                // unnormalised fp32 partial of key split blockIdx.z, merged by
-                // the combine; staged D/2 columns (RB bytes) at a time
+                // unnormalised fp32 partial (of key split blockIdx.z, or the
+                // private part), merged by the combine; staged D/2 columns
+                // (RB bytes) at a time
+                const int part = PREFIX ? (int)blockIdx.z : p.private_part;
 #pragma unroll
                 for (int hc = 0; hc < 2; ++hc) {
 #pragma unroll
@@ -666,11 +704,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                             *row_chunk(row, 8 * cc + v) = make_uint4(o[4 * v], o[4 * v + 1], o[4 * v + 2], o[4 * v + 3]);
                     }
                     drain([&](int i, int c) {
-                        const int64_t slot = row_idx[x * kRows + i] * p.parts_per_head + blockIdx.z;
+                        const int64_t slot = row_idx[x * kRows + i] * p.parts_per_head + part;
                         return reinterpret_cast<uint4 *>(p.o_part + slot * D + hc * (D / 2)) + c;
                     });
                 }
-                if (valid) p.ml_part[row_idx[x * kRows + row] * p.parts_per_head + blockIdx.z] = make_float2(m, l);
+                if (valid) p.ml_part[row_idx[x * kRows + row] * p.parts_per_head + part] = make_float2(m, l);
+                if constexpr (PART) {
+                    // the token's part counts for the combine: one private
+                    // part, and the prefix partials of its group
+                    if (valid && row % p.g == 0) {
+                        const int n_pre = blk_off > 0 ? min((blk_off + p.blocks_per_part - 1) / p.blocks_per_part,
+                                                            p.prefix_parts)
+                                                      : 0;
+                        p.nparts[(int64_t)(cu0 + q0 + qi) * p.Hkv + h] = 1 | (n_pre << 16);
+                    }
+                }
             }
         }
     }
@@ -681,21 +729,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_dealloc(tmem, kTmemCols);
     }
     if (threadIdx.x == 0 && *abort) latch_error(p.err, kDevTimeout);
+    if constexpr (PART) pdl_wait();
 }
 
 }  // namespace
 
-template <int D, bool PREFIX, bool TREE = false, bool FUSED = false>
+template <int D, bool PREFIX, bool TREE = false, bool FUSED = false, bool PART = false>
 static cudaError_t launch_tile_kernel(dim3 grid, const CUtensorMap &tk, const CUtensorMap &tv,
                                       const CUtensorMap &tkn, const CUtensorMap &tvn,
                                       const KernelParams &p, cudaStream_t stream) {
     // the d = 64 tiles are smaller; ask for the d = 128 footprint anyway so
     // one CTA owns an SM (its 512 TMEM columns never wait on a neighbour)
     static SmemLimit limit;
-    cudaError_t e = limit.ensure(reinterpret_cast<const void *>(attn_tile_kernel<D, PREFIX, TREE, FUSED>),
+    cudaError_t e = limit.ensure(reinterpret_cast<const void *>(attn_tile_kernel<D, PREFIX, TREE, FUSED, PART>),
                                  Layout<128>::kDynSmem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(attn_tile_kernel<D, PREFIX, TREE, FUSED>, grid, dim3(kThreads), Layout<128>::kDynSmem, stream,
+    return launch_pdl(attn_tile_kernel<D, PREFIX, TREE, FUSED, PART>, grid, dim3(kThreads), Layout<128>::kDynSmem, stream,
                       tk, tv, tkn, tvn, p);
 }
 
@@ -767,12 +816,57 @@ cudaError_t launch_decode_prefix(const DecodeLayout &L, const DecodeArgs &a,
     // keeps its successor until it exits: starting the split pass early
     // there measured much slower (l70b decode 345 -> 433 us per step).
     p.early_trigger = L.prefix_early;
+    p.group_row = a.group_row;
+    p.num_table_rows = a.num_table_rows;
     if (tr) tr->begin(kKernelDecodePrefix, stream);
     cudaError_t e = L.d == 128
                         ? launch_tile_kernel<128, true>(grid, *a.tmap_k, *a.tmap_v, *a.tmap_k, *a.tmap_v, p, stream)
                         : launch_tile_kernel<64, true>(grid, *a.tmap_k, *a.tmap_v, *a.tmap_k, *a.tmap_v, p, stream);
     if (tr) tr->end(kKernelDecodePrefix, stream);
     return e;
+}
+
+cudaError_t launch_verify_grouped(const DecodeLayout &L, const DecodeArgs &a, const PrefillArgs &pa,
+                                  const int32_t *request_group, cudaStream_t stream, Tracer *tr) {
+    // the shared prefixes, once per group: rows = draft tokens x heads
+    const bool prefix = L.prefix_parts > 0 && a.num_groups > 0 && request_group;
+    cudaError_t e = prefix ? launch_decode_prefix(L, a, pa.num_blocks_pool, stream, tr) : cudaSuccess;
+    if (e != cudaSuccess) return e;
+    // each request's private keys and drafts, under the draft masks, into
+    // the private part slot (beside the prefix pass when it leaves SMs free)
+    KernelParams p{};
+    p.q = static_cast<const uint16_t *>(pa.q);
+    p.cu_seqlens_q = pa.cu_seqlens_q;
+    p.context_lens = pa.context_lens;
+    p.block_table = pa.block_table;
+    p.max_blocks = pa.max_blocks;
+    p.Hq = pa.Hq; p.Hkv = pa.Hkv; p.g = pa.Hq / pa.Hkv; p.tpt = kRows / p.g;
+    p.num_blocks_pool = pa.num_blocks_pool;
+    p.scale_log2 = pa.scale_log2;
+    p.err = pa.err;
+    p.tree_mask = pa.tree_mask;
+    p.group_blocks = a.group_blocks;
+    p.request_group = prefix ? request_group : nullptr;   // no prefix pass: every key here
+    p.after_prefix = prefix ? 1 : 0;
+    p.blocks_per_part = L.prefix_blocks_per_part;
+    p.prefix_parts = L.prefix_parts;
+    p.parts_per_head = L.parts_per_head;
+    p.private_part = L.prefix_parts;
+    p.o_part = reinterpret_cast<float *>(static_cast<char *>(a.ws) + L.off_o);
+    p.ml_part = reinterpret_cast<float2 *>(static_cast<char *>(a.ws) + L.off_ml);
+    p.nparts = reinterpret_cast<int32_t *>(static_cast<char *>(a.ws) + L.off_nparts);
+    const int items = (pa.max_seqlen_q + 2 * p.tpt - 1) / (2 * p.tpt);
+    if (items <= 0 || pa.R <= 0) return cudaSuccess;
+    if (items > 65535) return cudaErrorInvalidConfiguration;
+    dim3 grid((unsigned)(pa.R * pa.Hkv), (unsigned)items);
+    if (tr) tr->begin(kKernelPrefill, stream);
+    e = pa.d == 128 ? launch_tile_kernel<128, false, true, false, true>(grid, *pa.tmap_k, *pa.tmap_v, *pa.tmap_k,
+                                                                         *pa.tmap_v, p, stream)
+                    : launch_tile_kernel<64, false, true, false, true>(grid, *pa.tmap_k, *pa.tmap_v, *pa.tmap_k,
+                                                                        *pa.tmap_v, p, stream);
+    if (tr) tr->end(kKernelPrefill, stream);
+    if (e != cudaSuccess) return e;
+    return launch_decode_combine(L, a, stream, tr);
 }
 
 }  // namespace pkv

@@ -45,6 +45,7 @@ EXPORTS = [
     "pkv_selftest_wait_timeout", "pkv_lora_dispatch", "pkv_check_block_table",
     "paged_attn_verify_tree", "pkv_tree_masks", "pkv_blocks_staging_size", "pkv_blocks_gather",
     "pkv_blocks_scatter", "pkv_lora_sgmv", "paged_attn_prefill_append",
+    "paged_attn_verify_tree_workspace_size", "paged_attn_verify_tree_grouped", "pkv_verify_groups_build",
 ]
 
 
@@ -71,6 +72,14 @@ class PrefixGroups(ctypes.Structure):
                 ("max_group_members", ctypes.c_int32), ("reserved", ctypes.c_int32),
                 ("group_start", ctypes.c_void_p), ("member_req", ctypes.c_void_p),
                 ("group_blocks", ctypes.c_void_p), ("group_of_req", ctypes.c_void_p)]
+
+
+class VerifyGroups(ctypes.Structure):
+    _fields_ = [("num_groups", ctypes.c_int32), ("max_group_blocks", ctypes.c_int32),
+                ("max_group_tokens", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("group_start", ctypes.c_void_p), ("member_token", ctypes.c_void_p),
+                ("group_blocks", ctypes.c_void_p), ("group_row", ctypes.c_void_p),
+                ("request_group", ctypes.c_void_p)]
 
 
 class StepLayout(ctypes.Structure):
@@ -134,6 +143,11 @@ def load(path: str | None = None):
         "pkv_check_block_table": [V, P, i32, i32, P, P],
         "paged_attn_verify_tree": [V, V, V, V, V, V, V, i32, i32, i32, i32, f32, V, V],
         "pkv_tree_masks": [P, P, i32, P],
+        "paged_attn_verify_tree_workspace_size": [V, i32, i32, i32, ctypes.POINTER(VerifyGroups),
+                                                  ctypes.POINTER(sz)],
+        "paged_attn_verify_tree_grouped": [V, V, V, V, V, V, V, i32, i32, i32, i32, i32, f32, V,
+                                           ctypes.POINTER(VerifyGroups), V, sz, V],
+        "pkv_verify_groups_build": [P, P, i32, i32, P, P, P, P],
         "pkv_blocks_staging_size": [V, i32, ctypes.POINTER(sz)],
         "paged_attn_prefill_append": [V, V, V, V, i32, V, V, V, V, V, i32, i32, i32, i32, f32, V],
         "pkv_lora_sgmv": [V, V, V, V, P, P, P, i32, i32, i32, i32, i32, i32, V, V, V],
@@ -410,6 +424,71 @@ def paged_attn_verify_tree(pool, q, out, lse, cu_seqlens_q, context_lens, block_
         pool, _dptr(q), _dptr(out), _dptr(lse), _dptr(cu_seqlens_q), _dptr(context_lens),
         _dptr(block_table), int(block_table.shape[1]), int(context_lens.shape[0]),
         int(max_seqlen_q), int(q.shape[1]), float(scale), _dptr(tree_mask), _stream(stream)))
+
+
+def pkv_verify_groups_build(cu_seqlens, request_group, num_groups: int) -> dict:
+    """Token groups of a verification batch (host): a dict with group_start,
+    member_token, group_row (int32 numpy arrays) and max_group_tokens."""
+    cu = np.ascontiguousarray(cu_seqlens, np.int32)
+    rg = np.ascontiguousarray(request_group, np.int32)
+    R = len(cu) - 1
+    _need(len(rg) == R, lambda: f"request_group must have {R} entries")
+    G = int(num_groups)
+    gstart = np.zeros(G + 1, np.int32)
+    members = np.zeros(max(int(cu[-1]), 1), np.int32)
+    grow = np.zeros(max(G, 1), np.int32)
+    mx = np.zeros(1, np.int32)
+    _check(load().pkv_verify_groups_build(_np_ptr(cu), _np_ptr(rg), R, G, _np_ptr(gstart), _np_ptr(members),
+                                          _np_ptr(grow), _np_ptr(mx)))
+    return dict(group_start=gstart, member_token=members[:int(gstart[G])], group_row=grow[:G],
+                max_group_tokens=int(mx[0]))
+
+
+def make_verify_groups(num_groups=0, max_group_blocks=0, max_group_tokens=0, group_start=None,
+                       member_token=None, group_blocks=None, group_row=None, request_group=None):
+    """The pkv_verify_groups descriptor over device int32 tensors (they must
+    outlive every call that takes it)."""
+    import torch
+    for name, t, n in (("group_start", group_start, num_groups + 1), ("member_token", member_token, 0),
+                       ("group_blocks", group_blocks, num_groups), ("group_row", group_row, num_groups),
+                       ("request_group", request_group, 0)):
+        if t is not None or num_groups > 0:
+            _check_tensor(name, t, torch.int32, 1)
+            _need(t.shape[0] >= n, lambda: f"{name} has {t.shape[0]} entries, {n} needed")
+    return VerifyGroups(int(num_groups), int(max_group_blocks), int(max_group_tokens), 0,
+                        _dptr(group_start), _dptr(member_token), _dptr(group_blocks), _dptr(group_row),
+                        _dptr(request_group))
+
+
+def paged_attn_verify_tree_workspace_size(pool, num_tokens: int, num_q_heads: int, max_blocks: int,
+                                          groups=None) -> int:
+    out = ctypes.c_size_t()
+    _check(load().paged_attn_verify_tree_workspace_size(
+        pool, int(num_tokens), int(num_q_heads), int(max_blocks),
+        ctypes.byref(groups) if groups is not None else None, ctypes.byref(out)))
+    return int(out.value)
+
+
+def paged_attn_verify_tree_grouped(pool, q, out, lse, cu_seqlens_q, context_lens, block_table,
+                                   max_seqlen_q: int, scale: float, tree_mask, groups, workspace,
+                                   stream=None):
+    """paged_attn_verify_tree with each group's shared prefix read once per
+    group (groups: make_verify_groups(...) or None)."""
+    import torch
+    _check_attn_args(pool, q, out, lse, context_lens, block_table, 0)
+    _need(tuple(out.shape) == tuple(q.shape), lambda: f"out must have q's shape {list(q.shape)}")
+    cs = _check_tensor("cu_seqlens_q", cu_seqlens_q, torch.int32, 1)
+    _need(cs[0] == context_lens.shape[0] + 1,
+          lambda: f"cu_seqlens_q must have {context_lens.shape[0] + 1} entries")
+    ms = _check_tensor("tree_mask", tree_mask, torch.int64, 1)
+    _need(ms[0] >= q.shape[0], lambda: f"tree_mask has {ms[0]} entries for {q.shape[0]} rows")
+    _check(load().paged_attn_verify_tree_grouped(
+        pool, _dptr(q), _dptr(out), _dptr(lse), _dptr(cu_seqlens_q), _dptr(context_lens),
+        _dptr(block_table), int(block_table.shape[1]), int(context_lens.shape[0]), int(q.shape[0]),
+        int(max_seqlen_q), int(q.shape[1]), float(scale), _dptr(tree_mask),
+        ctypes.byref(groups) if groups is not None else None, _dptr(workspace),
+        int(workspace.numel() * workspace.element_size()) if workspace is not None else 0,
+        _stream(stream)))
 
 
 def pkv_blocks_staging_size(pool, n: int) -> int:
