@@ -183,11 +183,23 @@ __device__ void build_plan(int32_t *P, int32_t *Ls, int32_t R, const int32_t *__
                            int32_t max_blocks, int32_t *max_n_out, int *err) {
     __shared__ int32_t warp_tot[kWarps];
     __shared__ int32_t warp_max[kWarps];
+    __shared__ int32_t s_gb[kThreads];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    // Up to kThreads groups: their shared block counts go to shared memory,
+    // loaded beside each thread's first request, so that no load waits on
+    // another.  More groups: a dependent load per request.
+    const bool gb_smem = num_groups <= kThreads;
+    if (num_groups > 0 && gb_smem && tid < num_groups) s_gb[tid] = __ldg(group_blocks + tid);
+    int32_t L0 = 0, gi0 = -1;
+    if (tid < R) {
+        L0 = __ldg(context_lens + tid);
+        if (num_groups > 0) gi0 = __ldg(group_of_req + tid);
+    }
+    __syncthreads();
     // private block counts, request r on thread r % kThreads (independent
     // loads, in flight together), kept in P for now
     for (int r = tid; r < R; r += kThreads) {
-        const int32_t L = __ldg(context_lens + r);
+        const int32_t L = r == tid ? L0 : __ldg(context_lens + r);
         int32_t nblk = (L + 15) >> 4;
         if (nblk > max_blocks) {   // context longer than the table row
             latch_error(err, kDevBounds);
@@ -195,8 +207,8 @@ __device__ void build_plan(int32_t *P, int32_t *Ls, int32_t R, const int32_t *__
         }
         int32_t sh = 0;
         if (num_groups > 0) {
-            const int32_t gi = __ldg(group_of_req + r);
-            if (gi >= 0 && gi < num_groups) sh = __ldg(group_blocks + gi);
+            const int32_t gi = r == tid ? gi0 : __ldg(group_of_req + r);
+            if (gi >= 0 && gi < num_groups) sh = gb_smem ? s_gb[gi] : __ldg(group_blocks + gi);
         }
         int32_t n = nblk - sh;
         if (L < 1 || n < 1 || sh < 0) {   // decode needs a private tail block holding the query
@@ -286,7 +298,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Without one, wait for the preceding kernel first.
     if (!after_prefix) pdl_wait();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (threadIdx.x == 0) abort_flag = 0;
+    {
+        // Warm L2 with the block table while the plan is built: its lines are
+        // split over the CTAs, one 128-byte line per thread and pass (tables
+        // up to 16 MiB).
+        const int64_t lines = min(((int64_t)lay.R * a.max_blocks * 4 + 127) >> 7, (int64_t)1 << 17);
+        const char *base = reinterpret_cast<const char *>(a.block_table);
+        for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < lines; i += (int64_t)gridDim.x * kThreads)
+            prefetch_l2(base + (i << 7));
+    }
+    if (threadIdx.x == 0) {
+        abort_flag = 0;
+        prefetch_tmap(&tmk);   // the descriptors are fetched while the plan is built
+        prefetch_tmap(&tmv);
+    }
     const uint32_t mybar = smem_u32(bars + warp * S);
     if (lane == 0) {
         for (int s = 0; s < S; ++s) mbar_init(mybar + 8 * s, 1);
@@ -306,6 +331,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (per < kMinBlocksPerPiece) per = kMinBlocksPerPiece;
     const int64_t gw = (int64_t)blockIdx.x * kWarps + warp;
     const int64_t x0 = gw * per, x1 = min(x0 + per, W);
+    // cost positions below 2^31 (every realistic batch) divide in 32 bits
+    const bool narrow = W < ((int64_t)1 << 31);
+    auto div_per = [&](int64_t v) -> int64_t {   // v >= 0
+        return narrow ? (int64_t)((uint32_t)v / (uint32_t)per) : v / per;
+    };
 
     if (x0 < x1) {
         float *o_part = reinterpret_cast<float *>(static_cast<char *>(a.ws) + lay.off_o);
@@ -328,13 +358,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if ((int64_t)P[mid] + (int64_t)c * mid <= xr) lo = mid; else hi = mid - 1;
             }
             const int32_t n0 = P[lo + 1] - P[lo];
-            seg_base = (int64_t)lo * Hkv + (x0 - (int64_t)Hkv * ((int64_t)P[lo] + (int64_t)c * lo)) / (n0 + c);
+            const int64_t off = x0 - (int64_t)Hkv * ((int64_t)P[lo] + (int64_t)c * lo);
+            seg_base = (int64_t)lo * Hkv + (narrow ? (int64_t)((uint32_t)off / (uint32_t)(n0 + c)) : off / (n0 + c));
         }
         int32_t pr = 0, ph = 0, plo = 0, phi = 0, psh = 0, pL = 0, pn = 0, ppart = 0, pnw = 0;
         auto fill_list = [&]() {
-            const int64_t sg = seg_base + lane;
-            pr = (int32_t)(sg / Hkv);
-            ph = (int32_t)(sg - (int64_t)pr * Hkv);
+            // segment ids stay below R * Hkv + 32 < 2^31
+            const int32_t sg = (int32_t)(seg_base + lane);
+            pr = (int32_t)((uint32_t)sg / (uint32_t)Hkv);
+            ph = sg - pr * Hkv;
             plo = phi = 0;
             if (pr < R) {
                 pn = P[pr + 1] - P[pr];
@@ -347,8 +379,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     pL = Ls ? Ls[pr] : __ldg(a.context_lens + pr);
                     const int32_t nblk = min((pL + 15) >> 4, a.max_blocks);
                     psh = max(nblk - pn, 0);
-                    ppart = lay.prefix_parts + (int32_t)(gw - b0 / per);
-                    const int32_t n_priv = (int32_t)((b0 + pn - 1) / per - b0 / per + 1);
+                    const int64_t w0 = div_per(b0);   // the warp whose range holds block 0
+                    ppart = lay.prefix_parts + (int32_t)(gw - w0);
+                    const int32_t n_priv = (int32_t)(div_per(b0 + pn - 1) - w0 + 1);
                     const int32_t n_pre = lay.prefix_parts > 0 && a.num_groups > 0
                                               ? min((psh + lay.prefix_blocks_per_part - 1) / lay.prefix_blocks_per_part,
                                                     lay.prefix_parts)
@@ -438,10 +471,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (first)   // the piece's g q-head rows, contiguous in q
                     bulk_load(qarea + (uint32_t)s * kQBytes,
                               static_cast<const uint16_t *>(a.q) + ((int64_t)cr * Hq + (int64_t)ch * g) * D, qbytes, bar);
+                // read once: marked first out of L2 (measured: the pass
+                // streams faster, and the shared-prefix pass beside it too)
+                const uint64_t pol = l2_evict_first_policy();
 #pragma unroll
                 for (int hf = 0; hf < kHalves; ++hf) {
-                    tma_load_4d(dst + hf * 2048, &tmk, hf * 64, 0, ch, phys, bar);
-                    tma_load_4d(dst + kTileBytes + hf * 2048, &tmv, hf * 64, 0, ch, phys, bar);
+                    tma_load_4d_hint(dst + hf * 2048, &tmk, hf * 64, 0, ch, phys, bar, pol);
+                    tma_load_4d_hint(dst + kTileBytes + hf * 2048, &tmv, hf * 64, 0, ch, phys, bar, pol);
                 }
             }
             __syncwarp();
@@ -449,10 +485,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             return true;
         };
 
-        if (lane == 0) {
-            prefetch_tmap(&tmk);
-            prefetch_tmap(&tmv);
-        }
         int64_t issued = 0;
         for (int s0 = 0; s0 < S && more; ++s0) {
             more = produce(s0);

@@ -36,6 +36,11 @@ __device__ __forceinline__ uint4 ldg16(const void *p) {
     return *reinterpret_cast<const uint4 *>(p);
 }
 
+// Bring the 128-byte line holding p into L2 (no register result, no wait).
+__device__ __forceinline__ void prefetch_l2(const void *p) {
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
 // D = A * B + C, m16n8k16, bf16 inputs, fp32 accumulate (warp-wide).
 __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a1,
                                                uint32_t a2, uint32_t a3, uint32_t b0,

@@ -314,11 +314,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_relinquish();
     }
     // global q row of every tile row (-1: no query), looked up once; the Q
-    // loads and the epilogue stores use this table
+    // loads and the epilogue stores use this table.  Thread t < 256 also
+    // copies tile row t of Q into shared memory (asynchronously, while the
+    // block ids below are read): K-major with the 128-byte swizzle, 16-byte
+    // chunk c of row i at chunk c ^ (i % 8) of its 128-byte row; rows
+    // without a query are zero-filled.
     int64_t *row_idx = reinterpret_cast<int64_t *>(smem + Ly::kRowIdx);
     if (threadIdx.x < 2 * kRows) {
         const int x = threadIdx.x >> 7, i = threadIdx.x & 127;
-        row_idx[threadIdx.x] = i < (x ? rows_b : rows_a) ? q_row(x * p.tpt + i / p.g, i % p.g) : -1;
+        const int64_t qr = i < (x ? rows_b : rows_a) ? q_row(x * p.tpt + i / p.g, i % p.g) : -1;
+        row_idx[threadIdx.x] = qr;
+        const uint16_t *src = p.q + (qr >= 0 ? qr : 0) * D;
+        const uint32_t dst_row = sb + Ly::kQ + x * Ly::kTile + i * 128;
+#pragma unroll
+        for (int c = 0; c < D / 8; ++c)
+            cp_async16(dst_row + (c >> 3) * Ly::kHalfBytes + (((c & 7) ^ (i & 7)) << 4), src + c * 8, qr >= 0);
     }
     // the item's physical block ids, checked once, for the producer
     int32_t *blk_ids = reinterpret_cast<int32_t *>(smem + Ly::kBlkIds);
@@ -332,7 +342,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncthreads();
     // The producer issues the K/V loads of the first two key tiles now, so
-    // that their latency overlaps the Q tile loads below.
+    // that their latency overlaps the Q copies still in flight.
     auto issue_kv = [&](int j, bool k_side) {
         const int s = j & 1;
         const int b0 = j * 8, nb = min(8, nblk - b0);
@@ -367,41 +377,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             issue_kv(j, false);
         }
     }
-    // Q tiles -> shared memory, K-major with the 128-byte swizzle (16-byte
-    // chunk c of row i goes to chunk c ^ (i % 8) of its 128-byte row).  All
-    // loads of a round are issued before its first store.
-    {
-        constexpr int kChunks = D / 8;
-        constexpr int kTotal = 2 * kRows * kChunks;
-        constexpr int kIters = (kTotal + kThreads - 1) / kThreads;
-        constexpr int kHalfIters = (kIters + 1) / 2;   // two rounds bound the registers held
-#pragma unroll
-        for (int round = 0; round < 2; ++round) {
-            uint4 v[kHalfIters];
-#pragma unroll
-            for (int k = 0; k < kHalfIters; ++k) {
-                const int idx = threadIdx.x + (round * kHalfIters + k) * kThreads;
-                const int row = idx / kChunks, c = idx % kChunks;
-                v[k] = make_uint4(0, 0, 0, 0);
-                if (idx < kTotal) {
-                    const int64_t qr = row_idx[row];
-                    if (qr >= 0) v[k] = ldg16(p.q + qr * D + c * 8);
-                }
-            }
-#pragma unroll
-            for (int k = 0; k < kHalfIters; ++k) {
-                const int idx = threadIdx.x + (round * kHalfIters + k) * kThreads;
-                if (idx < kTotal) {
-                    const int row = idx / kChunks, c = idx % kChunks;
-                    const int x = row >> 7, i = row & 127;
-                    const int half = c >> 3, cc = c & 7;
-                    *reinterpret_cast<uint4 *>(smem + Ly::kQ + x * Ly::kTile + half * Ly::kHalfBytes +
-                                               i * 128 + ((cc ^ (i & 7)) << 4)) = v[k];
-                }
-            }
-        }
-        fence_proxy_async_smem();
-    }
+    // the Q rows are in shared memory once every thread's copies have landed
+    cp_async_wait_all();
+    fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
