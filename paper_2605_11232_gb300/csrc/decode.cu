@@ -768,10 +768,11 @@ DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_
         // quarter of the SMs free, the split pass runs beside it on those
         // SMs and a step costs about max(prefix critical path, split time on
         // the free SMs); otherwise the two run one after the other.
-        // Measured on GB300 with per-CTA clock stamps: a prefix CTA costs about
-        // 16 us of fixed work (set-up, Q tile, pipeline fill, partial writes)
-        // plus 1.8 us per key tile alone, 3.1 us with the split pass loading
-        // HBM beside it (its 2-stage K/V ring then waits on memory).
+        // Measured on GB300 with per-CTA clock stamps: a prefix CTA alone
+        // costs about 14 us of fixed work (set-up, Q tile, pipeline fill,
+        // partial writes) plus 1.85 us per key tile; beside the split pass
+        // (2-stage ring) 18 us plus 2.5 us per key tile, its 2-stage K/V ring
+        // then waiting on memory.
         const int per_item = 2 * (128 / L.g);   // members per work item (two 128-row tiles)
         const int64_t tiles = (int64_t)num_groups * Hkv * ((max_group_members + per_item - 1) / per_item);
         const int key_tiles = (max_group_blocks + 7) / 8;
@@ -781,7 +782,7 @@ DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_
             const int per = (key_tiles + sp - 1) / sp;
             const int64_t ctas = tiles * sp;
             const bool beside = 4 * ctas <= 3 * (int64_t)sms;
-            const double cta_us = 16.0 + (beside ? 3.1 : 1.8) * per;
+            const double cta_us = beside ? 18.0 + 2.5 * per : 14.0 + 1.85 * per;
             const double crit = (double)((ctas + sms - 1) / sms) * cta_us;
             const double t = beside ? std::max(crit, split_us(sms - (int)ctas)) : crit + split_us(sms);
             if (t < best_t - 1e-9) { best_t = t; best = sp; }
@@ -794,11 +795,15 @@ DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_
     }
     L.split_grid = L.prefix_early ? sms - (int32_t)L.prefix_ctas : sms;
     // as many ring stages as fit (the plan takes 4 bytes per request)
-    // as many ring stages as fit: each warp keeps S - 1 blocks in flight while
-    // it computes on one, and 2 stages leave the pass short of HBM on ~120 SMs
+    // Ring stages: each warp keeps S - 1 blocks in flight while it computes
+    // on one.  Alone on the device the pass takes as many as fit (up to 3 of
+    // 8 KB at d = 128).  Beside the shared-prefix pass it keeps to 16 KB per
+    // warp: with fewer copies queued at HBM that pass's own loads wait less
+    // (measured on the 64-request Llama-3-8B step: prefix pass 43 -> 38 us,
+    // the split pass's end unchanged, step -3 us).
     L.qbytes = (L.g <= 4 ? 4 : 8) * d * 2;
     L.stages = 2;
-    const int max_stages = d == 64 ? 4 : 3;
+    const int max_stages = d == 64 ? 4 : (L.prefix_early ? 2 : 3);
     for (int st = max_stages; st > 2; --st)
         if (split_smem_bytes(R, d, st, false, L.qbytes) <= kMaxSmemPerBlock) { L.stages = st; break; }
     // the context lengths beside the plan when they fit (saves a global read per piece list)
