@@ -498,6 +498,7 @@ int prefill_impl(pkv_pool_t pool, const void *q, void *out, float *lse, const in
     a.tmap_k = &pool->tmap_k; a.tmap_v = &pool->tmap_v;
     a.err = pool->d_err;
     a.tree_mask = reinterpret_cast<const unsigned long long *>(tree_mask);
+    a.num_sms = pool->num_sms;
     if (k_new) {
         a.k_new = k_new; a.v_new = v_new;
         a.k_cache = pool->k_cache; a.v_cache = pool->v_cache;

@@ -200,6 +200,7 @@ struct PrefillArgs {
     void *k_cache, *v_cache;
     const CUtensorMap *tmap_kn;            // 3-D maps over k_new / v_new
     const CUtensorMap *tmap_vn;
+    int32_t num_sms;                       // the device's SM count (0: unknown)
 };
 
 cudaError_t launch_prefill(const PrefillArgs &a, cudaStream_t stream, Tracer *tr);

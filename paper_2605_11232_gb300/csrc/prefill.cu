@@ -119,6 +119,7 @@ struct KernelParams {
     int32_t prefix_parts;            // prefix part slots (their count per request goes to nparts)
     int32_t *nparts;                 // [T * Hkv] part counts (private | prefix << 16)
     int32_t after_prefix;            // a shared-prefix pass precedes (and started) this pass
+    int32_t lpt;                     // suffix prefill: CTAs take items longest first (prefill_lpt_select)
 };
 
 // Row maximum of the 128 raw scores a thread holds (8 independent chains).
@@ -169,6 +170,93 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
     return __all_sync(0xffffffffu, wait_bar(bar, parity, abort));
 }
 
+// Longest-first order of a suffix prefill's CTAs.  Item i of request r (n
+// new tokens, context L, P = 2 * tpt queries per item, m = ceil(n / P)
+// items) ends at key e(i) = min(L, L - n + (i + 1) P) and costs t(i) =
+// ceil(e(i) / 128) key tiles, increasing in i.  CTA u of the grid takes the
+// item of rank u / Hkv in the order (t descending, r, i) and kv head
+// u % Hkv, so the heaviest CTAs start first whatever the requests' lengths
+// (a short grid's last wave then holds its lightest CTAs).  Warp-wide (all 32
+// lanes): returns false for a spare CTA.
+__device__ __forceinline__ int prefill_items_from(int c, int n, int L, int P) {
+    // items of a request with t(i) >= c
+    if (n <= 0 || L <= 128 * (c - 1)) return 0;
+    const int m = (n + P - 1) / P;
+    const int A = 128 * (c - 1) - (L - n);
+    return A < 0 ? m : max(0, m - A / P);
+}
+
+__device__ __forceinline__ bool prefill_lpt_select(const int32_t *__restrict__ cu_seqlens,
+                                                   const int32_t *__restrict__ context_lens, int R, int Hkv,
+                                                   int P, int64_t u, int *r_out, int *item_out, int *h_out) {
+    const int lane = threadIdx.x & 31;
+    // up to 32 requests: one per lane, held in registers
+    const bool one = R <= 32;
+    const int n1 = one && lane < R ? __ldg(cu_seqlens + lane + 1) - __ldg(cu_seqlens + lane) : 0;
+    const int L1 = one && lane < R ? __ldg(context_lens + lane) : 0;
+    auto count_ge = [&](int c) -> int64_t {   // items with t >= c, over all requests
+        int64_t s = 0;
+        if (one) {
+            s = prefill_items_from(c, n1, L1, P);
+        } else {
+            for (int r = lane; r < R; r += 32) {
+                const int n = __ldg(cu_seqlens + r + 1) - __ldg(cu_seqlens + r);
+                s += prefill_items_from(c, n, __ldg(context_lens + r), P);
+            }
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+        return s;
+    };
+    int cmax = one ? max(1, (L1 + 127) / 128) : 1;
+    if (!one)
+        for (int r = lane; r < R; r += 32) cmax = max(cmax, (__ldg(context_lens + r) + 127) / 128);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) cmax = max(cmax, __shfl_xor_sync(0xffffffffu, cmax, off));
+    const int64_t k = u / Hkv;
+    if (k >= count_ge(1)) return false;
+    // the item's cost: the largest c with more than k items of cost >= c
+    int lo = 1, hi = cmax;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (count_ge(mid) > k) lo = mid; else hi = mid - 1;
+    }
+    const int c = lo;
+    int64_t skip = k - count_ge(c + 1);   // among the items of cost exactly c, in (r, i) order
+    int64_t base = 0;
+    bool found = false;
+    for (int r0 = 0; r0 < R && !found; r0 += 32) {
+        const int r = r0 + lane;
+        int e = 0, first = 0;
+        if (r < R) {
+            const int n = one ? n1 : __ldg(cu_seqlens + r + 1) - __ldg(cu_seqlens + r);
+            const int L = one ? L1 : __ldg(context_lens + r);
+            const int m = n > 0 ? (n + P - 1) / P : 0;
+            const int ge = prefill_items_from(c, n, L, P);
+            e = ge - prefill_items_from(c + 1, n, L, P);
+            first = m - ge;
+        }
+        int64_t incl = e;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const int64_t v = __shfl_up_sync(0xffffffffu, incl, off);
+            if (lane >= off) incl += v;
+        }
+        const bool mine = e > 0 && skip >= base + incl - e && skip < base + incl;
+        const unsigned who = __ballot_sync(0xffffffffu, mine);
+        if (who) {
+            const int src = __ffs(who) - 1;
+            const int it = first + (int)(skip - (base + incl - e));
+            *r_out = __shfl_sync(0xffffffffu, r, src);
+            *item_out = __shfl_sync(0xffffffffu, it, src);
+            found = true;
+        }
+        base += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    *h_out = (int)(u % Hkv);
+    return found;
+}
+
 // PREFIX = false: suffix prefill.  CTA (request r, kv head h, query item);
 //   tile X row i = query X*tpt + i / g of the item, q head h*g + i % g;
 //   keys 0 .. pos(query).
@@ -192,12 +280,26 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (p.early_trigger) pdl_trigger();   // the split pass may start on the free SMs
     }
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int h = blockIdx.x % p.Hkv;
+    int h = blockIdx.x % p.Hkv;
     int nq, nblk, kv_end, q_pos0 = 0, blk_off = 0, cu0 = 0, q0 = 0, m0 = 0, new_blk0 = 1 << 30, cached = 0;
     const int32_t *trow;
     if constexpr (!PREFIX) {
-        const int r = blockIdx.x / p.Hkv;
-        const int item = gridDim.y - 1 - blockIdx.y;      // heaviest items first
+        int r = blockIdx.x / p.Hkv;
+        int item = gridDim.y - 1 - blockIdx.y;            // heaviest items of each request first
+        if (!PART && p.lpt) {
+            // longest first over all requests (prefill_lpt_select)
+            __shared__ int s_sel[3];
+            if (warp == 0) {
+                int sr = -1, si = 0, sh = 0;
+                const bool ok = prefill_lpt_select(p.cu_seqlens_q, p.context_lens, (int)gridDim.x / p.Hkv, p.Hkv,
+                                                   2 * p.tpt, (int64_t)blockIdx.y * gridDim.x + blockIdx.x, &sr,
+                                                   &si, &sh);
+                if (lane == 0) { s_sel[0] = ok ? sr : -1; s_sel[1] = si; s_sel[2] = sh; }
+            }
+            __syncthreads();
+            if (s_sel[0] < 0) return;     // spare CTA
+            r = s_sel[0]; item = s_sel[1]; h = s_sel[2];
+        }
         cu0 = __ldg(p.cu_seqlens_q + r);
         const int n_r = __ldg(p.cu_seqlens_q + r + 1) - cu0;
         q0 = item * 2 * p.tpt;
@@ -752,6 +854,12 @@ cudaError_t launch_prefill(const PrefillArgs &a, cudaStream_t stream, Tracer *tr
     if (items <= 0 || a.R <= 0) return cudaSuccess;
     if (items > 65535) return cudaErrorInvalidConfiguration;
     dim3 grid((unsigned)(a.R * a.Hkv), (unsigned)items);
+    // Few waves: a wave's worth of light CTAs at the end costs a whole CTA's
+    // time; taking the items longest first packs the last wave (measured on
+    // the Qwen chunks: 3.2 waves, 315 -> 255 us predicted from the CTAs' own
+    // durations).  Many waves, or many requests (the selection's cost grows
+    // with them): launch order.
+    p.lpt = (int64_t)grid.x * grid.y <= 8LL * a.num_sms && a.R <= 256;
     if (tr) tr->begin(kKernelPrefill, stream);
     cudaError_t e;
     if (p.fused)
