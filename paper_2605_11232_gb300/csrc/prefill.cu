@@ -598,13 +598,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                 fence_proxy_async_smem();
             }
             const bool more = j + 1 < nkt;
+            // tile A: P.V(j) as soon as P is ready, then Q.K(j+1) into the S
+            // it just consumed once K(j+1) has landed (measured: K(j+1)
+            // arrives up to ~0.5 us after P(j); waiting for it before P.V(j)
+            // kept the tensor core idle for that long every key tile)
+            if (!wait_bar(sb + Ly::kPFull, j & 1, abort)) { ok = false; break; }
+            issue_pv(0, j);
             if (more && !wait_bar(sb + Ly::kKFull + 8 * (s ^ 1), ((j + 1) >> 1) & 1, abort)) {
                 ok = false;
                 break;
             }
-            // tile A: P.V(j), then Q.K(j+1) into the S it just consumed
-            if (!wait_bar(sb + Ly::kPFull, j & 1, abort)) { ok = false; break; }
-            issue_pv(0, j);
             if (more) issue_qk(0, j + 1);
             if (has_b) {
                 if (!wait_bar(sb + Ly::kPFull + 8, j & 1, abort)) { ok = false; break; }
