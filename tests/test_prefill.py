@@ -300,3 +300,21 @@ def test_prefill_longest_item_and_empty_request():
     out, lse = run_prefill(b)
     compare(b, out, lse, [0, 2])
     b.close()
+
+
+@pytest.mark.parametrize("R", [32, 33, 70])
+def test_prefill_many_requests_longest_first(R):
+    """A short grid (a few waves) takes its items longest first over all
+    requests; with more than 32 requests the selection walks them in chunks
+    of 32.  Ragged suffixes (some empty), ragged cached contexts: every row
+    against the oracle."""
+    need_gpu()
+    rng = np.random.default_rng(R)
+    new = [int(x) for x in rng.choice([0, 1, 7, 33, 64, 65, 130, 200], R)]
+    cached = [int(x) for x in rng.integers(1, 600, R)]
+    w = make_workload("custom", seed=R, custom=dict(Hq=8, Hkv=2, d=64, prefix_lens=[], group=[-1] * R,
+                                                   cached=cached, new=new, decode=[False] * R))
+    b = B.build_batch(w, poison=True)
+    out, lse = run_prefill(b)
+    compare(b, out, lse, [r for r in range(R) if new[r] > 0])
+    b.close()

@@ -270,3 +270,42 @@ def test_verify_grouped_short_cache_latches_bounds():
     B.run_verify_grouped(b, out, None, torch.from_numpy(masks).cuda(), vg, ws, max(ks))
     assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_ERR_DEVICE_BOUNDS
     b.close()
+
+
+@pytest.mark.gpu
+def test_verify_grouped_two_groups():
+    """Two groups over prefixes of different lengths (512 and 256 tokens) and
+    ungrouped requests: every draft row against the fp64 tree oracle."""
+    from paper_2605_11232_gb300 import batch as B
+    from paper_2605_11232_gb300.workloads import make_workload
+    need_gpu()
+    rng = np.random.default_rng(9)
+    R = 10
+    ks = [3, 8, 1, 16, 5, 64, 2, 9, 12, 4]
+    grp = [0, 1, -1, 0, 1, 0, 1, -1, 0, 1]
+    plen = [512, 256]
+    cached = [int(rng.integers(1, 20 * 16)) + (plen[g0] if g0 >= 0 else 0) for g0 in grp]
+    w = make_workload("custom", seed=9, custom=dict(
+        Hq=32, Hkv=8, d=128, prefix_lens=plen, group=grp, cached=cached, new=ks, decode=[False] * R))
+    parents = [_random_parents(rng, k) for k in ks]
+    cu = np.concatenate([[0], np.cumsum(ks)]).astype(np.int32)
+    masks = pkv.pkv_tree_masks(np.concatenate(parents).astype(np.int32), cu)
+    b = B.build_batch(w, poison=True)
+    B.run_write(b)
+    T = int(cu[-1])
+    vg, keep = B.verify_groups(b)
+    ws = B.verify_workspace(b, vg)
+    out = torch.full((T, 32, 128), float("nan"), dtype=torch.bfloat16, device="cuda")
+    lse = torch.full((T, 32), float("nan"), dtype=torch.float32, device="cuda")
+    B.run_verify_grouped(b, out, lse, torch.from_numpy(masks).cuda(), vg, ws, max(ks))
+    assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_OK
+    errs, lerrs = [], []
+    for r in range(R):
+        kr, vr = w.request_kv(r)
+        o_ref, l_ref = TV.tree_verify_attention(_bits(w.request_q(r)), _bits(kr), _bits(vr), parents[r], w.scale)
+        a, e = int(cu[r]), int(cu[r + 1])
+        errs.append(np.abs(out[a:e].float().cpu().numpy().astype(np.float64) - o_ref).ravel())
+        lerrs.append(np.abs(lse[a:e].cpu().numpy().astype(np.float64) - l_ref).ravel())
+    err, lerr = np.concatenate(errs), np.concatenate(lerrs)
+    assert err.max() <= MAX_ABS and err.mean() <= MEAN_ABS and lerr.max() <= LSE_ABS
+    b.close()
