@@ -419,7 +419,9 @@ int paged_attn_verify_tree_workspace_size(pkv_pool_t pool, int32_t num_tokens, i
  * keys after them (its private context and its drafts, under the draft
  * masks), and the log-sum-exp merge of the two.  Same result as
  * paged_attn_verify_tree up to rounding (the merge of two partial softmaxes).
- *  num_tokens: cu_seqlens_q[num_requests] (host).  groups: as above, or NULL.
+ *  num_tokens: cu_seqlens_q[num_requests] (host); the workspace holds
+ *  partials for that many rows, and a request whose rows reach past it is
+ *  skipped and latches DEVICE_BOUNDS.  groups: as above, or NULL.
  *  A grouped request's cached part, context_lens[r] - n_r, must cover its
  *  group's blocks (else it latches DEVICE_BOUNDS and its outputs are
  *  undefined).

@@ -118,6 +118,7 @@ struct KernelParams {
     int32_t private_part;
     int32_t prefix_parts;            // prefix part slots (their count per request goes to nparts)
     int32_t *nparts;                 // [T * Hkv] part counts (private | prefix << 16)
+    int32_t num_rows;                // T: tokens the workspace holds partials for
     int32_t after_prefix;            // a shared-prefix pass precedes (and started) this pass
     int32_t lpt;                     // suffix prefill: CTAs take items longest first (prefill_lpt_select)
 };
@@ -330,7 +331,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             // here on count from there
             const int grp = p.request_group ? __ldg(p.request_group + r) : -1;
             blk_off = grp >= 0 ? __ldg(p.group_blocks + grp) : 0;
-            if (blk_off < 0 || blk_off * 16 > q_pos0) {
+            // the partials of rows cu0 .. cu0 + n_r - 1 must lie in the
+            // workspace, sized for num_rows tokens
+            if (blk_off < 0 || blk_off * 16 > q_pos0 || cu0 < 0 || cu0 + n_r > p.num_rows) {
                 if (threadIdx.x == 0) latch_error(p.err, kDevBounds);
                 pdl_wait();
                 return;
@@ -944,6 +947,7 @@ cudaError_t launch_verify_grouped(const DecodeLayout &L, const DecodeArgs &a, co
     p.o_part = reinterpret_cast<float *>(static_cast<char *>(a.ws) + L.off_o);
     p.ml_part = reinterpret_cast<float2 *>(static_cast<char *>(a.ws) + L.off_ml);
     p.nparts = reinterpret_cast<int32_t *>(static_cast<char *>(a.ws) + L.off_nparts);
+    p.num_rows = L.R;
     const int items = (pa.max_seqlen_q + 2 * p.tpt - 1) / (2 * p.tpt);
     if (items <= 0 || pa.R <= 0) return cudaSuccess;
     if (items > 65535) return cudaErrorInvalidConfiguration;

@@ -309,3 +309,25 @@ def test_verify_grouped_two_groups():
     err, lerr = np.concatenate(errs), np.concatenate(lerrs)
     assert err.max() <= MAX_ABS and err.mean() <= MEAN_ABS and lerr.max() <= LSE_ABS
     b.close()
+
+
+@pytest.mark.gpu
+def test_verify_grouped_token_count_below_cu_seqlens_stays_in_workspace():
+    """A num_tokens smaller than cu_seqlens_q[R] (the workspace sized for it):
+    the rows past it latch DEVICE_BOUNDS and nothing is written past the
+    workspace (a canary after it keeps its bytes)."""
+    from paper_2605_11232_gb300 import batch as B
+    need_gpu()
+    w, b, parents, cu, masks, ks = _tree_batch(128, 32, 8, 4)
+    vg, keep = B.verify_groups(b)
+    T = int(cu[-1])
+    T_small = int(cu[len(ks) // 2])          # half the requests' tokens
+    need = pkv.paged_attn_verify_tree_workspace_size(b.pool, T_small, 32, b.table.shape[1], vg)
+    buf = torch.full((need + (1 << 20),), 0x5A, dtype=torch.uint8, device="cuda")
+    out = torch.empty((T, 32, 128), dtype=torch.bfloat16, device="cuda")
+    m = torch.from_numpy(masks).cuda()
+    pkv.paged_attn_verify_tree_grouped(b.pool, b.q[:T_small], out[:T_small], None, b.cu_pre, b.context_lens,
+                                       b.table, max(ks), w.scale, m, vg, buf[:need])
+    assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_ERR_DEVICE_BOUNDS
+    assert bool((buf[need:] == 0x5A).all())
+    b.close()
