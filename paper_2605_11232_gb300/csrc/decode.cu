@@ -769,9 +769,9 @@ DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_
         // SMs and a step costs about max(prefix critical path, split time on
         // the free SMs); otherwise the two run one after the other.
         // Measured on GB300 with per-CTA clock stamps: a prefix CTA alone
-        // costs about 14 us of fixed work (set-up, Q tile, pipeline fill,
-        // partial writes) plus 1.85 us per key tile; beside the split pass
-        // (2-stage ring) 18 us plus 2.5 us per key tile, its 2-stage K/V ring
+        // costs about 11.5 us of fixed work (set-up, Q tile, pipeline fill,
+        // partial writes) plus 1.7 us per key tile; beside the split pass
+        // (2-stage ring) 13 us plus 2.2 us per key tile, its 2-stage K/V ring
         // then waiting on memory.
         const int per_item = 2 * (128 / L.g);   // members per work item (two 128-row tiles)
         const int64_t tiles = (int64_t)num_groups * Hkv * ((max_group_members + per_item - 1) / per_item);
@@ -782,7 +782,7 @@ DecodeLayout decode_layout(int32_t R, int32_t Hq, int32_t Hkv, int32_t d, int32_
             const int per = (key_tiles + sp - 1) / sp;
             const int64_t ctas = tiles * sp;
             const bool beside = 4 * ctas <= 3 * (int64_t)sms;
-            const double cta_us = beside ? 18.0 + 2.5 * per : 14.0 + 1.85 * per;
+            const double cta_us = beside ? 13.0 + 2.2 * per : 11.5 + 1.7 * per;
             const double crit = (double)((ctas + sms - 1) / sms) * cta_us;
             const double t = beside ? std::max(crit, split_us(sms - (int)ctas)) : crit + split_us(sms);
             if (t < best_t - 1e-9) { best_t = t; best = sp; }
