@@ -281,6 +281,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     if constexpr (PREFIX) {
         if (p.early_trigger) pdl_trigger();   // the split pass may start on the free SMs
     }
+    // A prefix pass that fills the device lets the split pass launch once
+    // every CTA is past its key-tile loop: the split pass's CTAs then take
+    // SMs as this pass's CTAs leave (it reads nothing this pass writes, and
+    // waits for it before exiting).  Every thread calls this once.
+    auto late_trigger = [&]() {
+        if constexpr (PREFIX) {
+            if (!p.early_trigger) pdl_trigger();
+        }
+    };
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int h = blockIdx.x % p.Hkv;
     int nq, nblk, kv_end, q_pos0 = 0, blk_off = 0, cu0 = 0, q0 = 0, m0 = 0, new_blk0 = 1 << 30, cached = 0;
@@ -656,6 +665,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
       }
+      late_trigger();
     } else {
         // ------------------------------------------------------------ softmax
         const int x = (warp - 4) >> 2;                // tile A (warps 4-7) or B (8-11)
@@ -734,6 +744,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_before();
             mbar_arrive(sb + Ly::kPFull + 8 * x);
         }
+        late_trigger();   // before the epilogue's partial writes
         if (ok && warp_wait(sb + Ly::kODone + 8 * x, 0, abort)) {
             tc_fence_after();
             // Epilogue through shared memory: every MMA reading Q_X has
