@@ -14,7 +14,8 @@
 // per segment it touches.  The combine kernel merges a head's partials with
 // log-sum-exp weights.  The grid covers the SMs the shared-prefix pass leaves
 // free (all of them without one), so all warps start together and end
-// together.
+// together; beside a prefix pass that fills the device it covers every SM,
+// its CTAs starting as the prefix pass's CTAs exit.
 //
 // Data path (per warp).  The (block, kv head) K and V tiles of the warp's
 // range are copied by TMA, with the 128-byte swizzle, into a ring of stages
@@ -838,8 +839,9 @@ static cudaError_t launch_decode_t(const DecodeLayout &L, const DecodeArgs &a, i
         if (e != cudaSuccess) return e;
     }
     if (tr) tr->begin(kKernelDecodeSplit, stream);
-    // the split pass runs beside an early-triggering prefix pass on the SMs
-    // it leaves free, after a late-triggering one on all of them
+    // the split pass runs beside the prefix pass: on the SMs that pass leaves
+    // free when they are a quarter of the device, otherwise on every SM (its
+    // CTAs take the SMs the prefix pass leaves idle, then those its CTAs free)
     const int grid = prefix ? L.split_grid : L.sms;
     cudaError_t e = launch_pdl(decode_split_kernel<D>, dim3(grid), dim3(kThreads), L.split_smem, stream,
                                *a.tmap_k, *a.tmap_v, a, L, num_blocks_pool, prefix ? 1 : 0);

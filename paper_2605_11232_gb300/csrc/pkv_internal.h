@@ -105,8 +105,8 @@ struct DecodeLayout {
     int32_t prefix_parts;        // prefix-pass part slots per head (0 without groups)
     int32_t prefix_blocks_per_part;
     int64_t prefix_ctas;         // CTAs of the prefix pass (0 without groups)
-    int32_t prefix_early;        // the prefix pass lets the split pass start beside it
-    int32_t split_grid;          // split-pass CTAs beside an early prefix pass
+    int32_t prefix_early;        // the prefix pass leaves a quarter of the SMs to the split pass
+    int32_t split_grid;          // split-pass CTAs beside such a prefix pass (sms - prefix_ctas)
     int32_t stages;              // ring stages per warp of the split pass
     int32_t qbytes;              // bytes of a stage's Q area (4 or 8 head rows)
     int32_t lens_in_smem;        // the split pass keeps the context lengths in shared memory
