@@ -240,6 +240,28 @@ def test_grouped_members_need_not_be_contiguous():
     b.close()
 
 
+@pytest.mark.parametrize("append", [False, True])
+def test_prefix_pass_larger_than_the_device(append):
+    """40 groups of 3 members over 8 kv heads: 320 shared-prefix CTAs (one key
+    split each), three waves on a 152-SM device, so the split pass (launched
+    once every prefix CTA has started, on all SMs) takes SMs only as
+    last-wave prefix CTAs exit.  Ragged prefixes (768-1024 tokens) and 8 requests outside any
+    group; every request against the oracle."""
+    need_gpu()
+    G, M = 40, 3
+    prefix_lens = [1024 - 64 * (g % 5) for g in range(G)]
+    group = [g for g in range(G) for _ in range(M)] + [-1] * 8
+    cached = [(prefix_lens[g] if g >= 0 else 0) + 1 + (37 * i) % 300 for i, g in enumerate(group)]
+    R = len(group)
+    w = make_workload("custom", custom=dict(Hq=32, Hkv=8, d=128, prefix_lens=prefix_lens, group=group,
+                                          cached=cached, new=[1] * R, decode=[True] * R))
+    b = B.build_batch(w, poison=True)
+    out, lse = (run_decode_append if append else run_decode)(b, use_groups=True)
+    assert torch.isfinite(out.float()).all()
+    compare(b, out, lse, range(R), threads=16)
+    b.close()
+
+
 def test_single_key_returns_value():
     """A context of one token returns that token's V (weight exactly 1)."""
     need_gpu()
