@@ -6,14 +6,15 @@
 //     y_t = W x_t + s_a B_a (A_a x_t)      (a = -1: y_t = W x_t)
 // One CTA computes a 128-row x 256-column tile of y for one segment:
 //   - a TMA producer thread streams 64-wide K chunks of the token rows X, of
-//     W's 256 output rows and of A_a's rank rows into a 3-stage ring
+//     W's 256 output rows and of A_a's rank rows into a 4-stage ring
 //     (128-byte swizzle);
 //   - one MMA thread issues Y += X.W^T (N = 256) and U += X.A_a^T (N = rank)
 //     into tensor memory for each chunk;
 //   - after the last chunk the 128 threads (thread = row) scale U by s_a,
-//     round it to bf16 and stage it in shared memory beside B_a's 256 rows,
-//     and the MMA thread adds Y += U.B_a^T (K = rank, padded to 64 with
-//     zeros);
+//     round it to bf16 and stage it in shared memory beside B_a's 256 rows
+//     (held in registers since the start; both go where the ring's first
+//     stage was), and the MMA thread adds Y += U.B_a^T (K = rank, padded to
+//     64 with zeros);
 //   - the epilogue rounds Y to bf16 and stores the segment's rows.
 // The low-rank update rides on the base GEMM's tile: x is read once for
 // both products and the delta never leaves the SM.
@@ -36,18 +37,23 @@ namespace {
 using namespace tc;
 
 constexpr int kThreads = 128;
-constexpr int kBM = 128, kBN = 256, kBK = 64, kStages = 3;
+constexpr int kBM = 128, kBN = 256, kBK = 64, kStages = 4;
 constexpr int kMaxRank = 64;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr uint64_t kDrainLimitNs = 200000000ull;
-// shared memory: stages of [X 128 x 64 | W 256 x 64 | A 64 x 64], then U
-// (128 x 64) and B_a's tile (256 x 64), all bf16 K-major, 128-byte swizzle
+// shared memory: stages of [X 128 x 64 | W 256 x 64 | A 64 x 64], all bf16
+// K-major, 128-byte swizzle.  Once every MMA of the main loop is done, U
+// (128 x 64) takes stage 0's X part and B_a's tile (256 x 64) its W part.
+// Four stages against three with U and B_a in their own space (the ring's
+// bytes in flight then cover about 1.3 us of MMA work instead of 1 us):
+// Case C1 595 -> 541 us, a 64-prompt request 2.94 -> 2.70 ms.
 constexpr int kXBytes = kBM * kBK * 2, kWBytes = kBN * kBK * 2, kABytes = kMaxRank * kBK * 2;
 constexpr int kStageBytes = kXBytes + kWBytes + kABytes;
-constexpr int kUOff = kStages * kStageBytes;
-constexpr int kBtOff = kUOff + kBM * kBK * 2;
-constexpr int kBarOff = kBtOff + kBN * kBK * 2;   // full[3] empty[3] done1 done2
-constexpr int kSmemBytes = kBarOff + 8 * 8 + 16 + 1024;
+constexpr int kUOff = 0;
+constexpr int kBtOff = kXBytes;
+static_assert(kBM * kBK * 2 <= kXBytes && kBN * kBK * 2 <= kWBytes, "U and B_a fit stage 0");
+constexpr int kBarOff = kStages * kStageBytes;   // full[kStages] empty[kStages] done1 done2
+constexpr int kSmemBytes = kBarOff + 8 * (2 * kStages + 2) + 16 + 1024;
 static_assert(kSmemBytes <= 227 * 1024, "shared memory of the LoRA tile");
 
 struct Tile {
@@ -80,8 +86,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int n0 = blockIdx.x * kBN;
     const bool lora = tile.adapter >= 0;
     const int nk = d_in / kBK;
-    const uint32_t bar_full = sb + kBarOff, bar_empty = bar_full + 24, bar_done1 = bar_full + 48,
-                   bar_done2 = bar_full + 56;
+    const uint32_t bar_full = sb + kBarOff, bar_empty = bar_full + 8 * kStages,
+                   bar_done1 = bar_full + 16 * kStages, bar_done2 = bar_done1 + 8;
     if (t == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(bar_full + 8 * s, 1);
@@ -96,18 +102,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_alloc(smem_u32(&tmem_slot), 512);   // Y in columns [0, 256), U in [256, 256 + rank)
         tmem_relinquish();
     }
-    if (lora) {
-        // B_a's rows n0 .. n0 + 255 (rank values each), K-major with the
-        // 128-byte swizzle, zero past the rank
-        const int cpr = rank / 8;
-        for (int i = t; i < kBN * 8; i += kThreads) {
-            const int row = i >> 3, c = i & 7;
-            uint4 v = make_uint4(0, 0, 0, 0);
-            if (c < cpr)
-                v = ldg16(lora_b + ((int64_t)tile.adapter * d_out + n0 + row) * rank + c * 8);
-            *reinterpret_cast<uint4 *>(smem + kBtOff + sw128(row, c)) = v;
+    // B_a's rows n0 .. n0 + 255 (rank values each), zero past the rank:
+    // thread t holds 16-byte chunk t % 8 of rows t / 8 + 16 i, in flight
+    // during the main loop and staged once the ring is free
+    constexpr int kBRegs = kBN * 8 / kThreads;
+    uint4 breg[kBRegs];
+    {
+        const int c = t & 7;
+#pragma unroll
+        for (int i = 0; i < kBRegs; ++i) {
+            const int row = (t >> 3) + i * (kThreads / 8);
+            breg[i] = (lora && c < rank / 8)
+                          ? ldg16(lora_b + ((int64_t)tile.adapter * d_out + n0 + row) * rank + c * 8)
+                          : make_uint4(0, 0, 0, 0);
         }
-        fence_proxy_async_smem();
     }
     tc_fence_before();
     __syncthreads();
@@ -182,6 +190,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             *reinterpret_cast<uint4 *>(smem + kUOff + sw128(t, c)) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
         }
+#pragma unroll
+        for (int i = 0; i < kBRegs; ++i)
+            *reinterpret_cast<uint4 *>(smem + kBtOff + sw128((t >> 3) + i * (kThreads / 8), t & 7)) = breg[i];
         fence_proxy_async_smem();
     }
     tc_fence_before();
