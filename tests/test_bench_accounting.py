@@ -40,3 +40,21 @@ def test_summary_reports_algorithmic_and_logical_rates():
     out = bench.summarize(res, (6774.6, 1934.6, 1725.0, "measured"))
     assert out["decode_logical_gbs"] > out["decode_hbm_gbs"] > 0
     assert abs(out["decode_hbm_gbs"] - (res["dec_bytes"] + res["wr_bytes"]) / 0.05e-3 / 1e9) < 1e-6
+
+
+def test_mixed_step_rates_use_the_decode_subsets_own_time():
+    """A step with prefill and decode requests: the decode bytes are set
+    against the decode subset timed alone (its kernels overlapping), not the
+    whole step nor the sum of traced kernel times; prefill TFLOP/s against
+    the traced prefill kernel."""
+    w = make_workload("qwen_mixed", values=False)
+    trace = {"decode_split": (3, 0.180), "decode_prefix": (3, 0.105), "decode_combine": (3, 0.030),
+             "prefill": (3, 0.750)}
+    res = dict(step_ms=[0.35] * 3, warm_ms=[0.35] * 3, dec_ms=[0.09, 0.09, 0.09], trace=trace, Rd=256, Rp=8,
+               dec_bytes=3.6e8, dec_logical=2.4e9, wr_bytes=1.0e6, pre_flops=2.6e11, groups=True)
+    out = bench.summarize(res, (6774.6, 1934.6, 1725.0, "measured"))
+    assert abs(out["decode_us_per_step"] - 90.0) < 1e-9
+    assert abs(out["decode_hbm_gbs"] - 3.6e8 / 90e-6 / 1e9) < 1e-6
+    assert abs(out["decode_kernels_sum_us"] - 1e3 * (0.180 + 0.105 + 0.030) / 3) < 1e-9
+    assert abs(out["prefill_tflops"] - 2.6e11 / 0.250e-3 / 1e12) < 1e-9
+    assert "alone" in out["decode_basis"]
