@@ -191,10 +191,14 @@ __device__ __forceinline__ bool prefill_lpt_select(const int32_t *__restrict__ c
                                                    const int32_t *__restrict__ context_lens, int R, int Hkv,
                                                    int P, int64_t u, int *r_out, int *item_out, int *h_out) {
     const int lane = threadIdx.x & 31;
+    // a request's keys are taken as at least its new tokens, so that every
+    // item of a request with new tokens is scheduled even where the lengths
+    // are inconsistent (the kernel then latches DEVICE_BOUNDS for it)
+    auto keys_of = [&](int r, int n) -> int { return max(__ldg(context_lens + r), n); };
     // up to 32 requests: one per lane, held in registers
     const bool one = R <= 32;
     const int n1 = one && lane < R ? __ldg(cu_seqlens + lane + 1) - __ldg(cu_seqlens + lane) : 0;
-    const int L1 = one && lane < R ? __ldg(context_lens + lane) : 0;
+    const int L1 = one && lane < R ? keys_of(lane, n1) : 0;
     auto count_ge = [&](int c) -> int64_t {   // items with t >= c, over all requests
         int64_t s = 0;
         if (one) {
@@ -202,7 +206,7 @@ __device__ __forceinline__ bool prefill_lpt_select(const int32_t *__restrict__ c
         } else {
             for (int r = lane; r < R; r += 32) {
                 const int n = __ldg(cu_seqlens + r + 1) - __ldg(cu_seqlens + r);
-                s += prefill_items_from(c, n, __ldg(context_lens + r), P);
+                s += prefill_items_from(c, n, keys_of(r, n), P);
             }
         }
 #pragma unroll
@@ -211,7 +215,8 @@ __device__ __forceinline__ bool prefill_lpt_select(const int32_t *__restrict__ c
     };
     int cmax = one ? max(1, (L1 + 127) / 128) : 1;
     if (!one)
-        for (int r = lane; r < R; r += 32) cmax = max(cmax, (__ldg(context_lens + r) + 127) / 128);
+        for (int r = lane; r < R; r += 32)
+            cmax = max(cmax, (keys_of(r, __ldg(cu_seqlens + r + 1) - __ldg(cu_seqlens + r)) + 127) / 128);
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) cmax = max(cmax, __shfl_xor_sync(0xffffffffu, cmax, off));
     const int64_t k = u / Hkv;
@@ -231,7 +236,7 @@ __device__ __forceinline__ bool prefill_lpt_select(const int32_t *__restrict__ c
         int e = 0, first = 0;
         if (r < R) {
             const int n = one ? n1 : __ldg(cu_seqlens + r + 1) - __ldg(cu_seqlens + r);
-            const int L = one ? L1 : __ldg(context_lens + r);
+            const int L = one ? L1 : keys_of(r, n);
             const int m = n > 0 ? (n + P - 1) / P : 0;
             const int ge = prefill_items_from(c, n, L, P);
             e = ge - prefill_items_from(c + 1, n, L, P);

@@ -180,6 +180,25 @@ def test_prefill_append_needs_block_aligned_cache():
     b.close()
 
 
+def test_prefill_context_shorter_than_its_new_tokens_latches_bounds():
+    """A request whose context length (a device array) is below its own
+    new-token count is refused on the device.  In the longest-first order of
+    a short grid its items are still given CTAs, so the error is latched
+    rather than the rows skipped unnoticed; the other requests are computed."""
+    need_gpu()
+    w = make_workload("custom", seed=43, custom=dict(Hq=8, Hkv=2, d=128, prefix_lens=[], group=[-1] * 3,
+                                                   cached=[64, 80, 96], new=[40, 30, 20], decode=[False] * 3))
+    b = B.build_batch(w, poison=True)
+    B.run_write(b)
+    out = torch.full((w.num_new_tokens, 8, 128), float("nan"), dtype=torch.bfloat16, device="cuda")
+    b.context_lens[1] = 0                               # request 1: no context for its 30 new tokens
+    B.run_prefill(b, out, None)
+    assert pkv.pkv_check_device_errors(b.pool) == pkv.PKV_ERR_DEVICE_BOUNDS
+    assert bool(torch.isnan(out[40:70].float()).all())
+    compare(b, out, None, [0, 2])
+    b.close()
+
+
 def test_prefill_refuses_tables_wider_than_its_limit():
     """A work item's block ids are staged in shared memory, 2048 of them at
     most: a table wider than that is refused on the host (UNSUPPORTED) before
