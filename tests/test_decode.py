@@ -262,6 +262,28 @@ def test_prefix_pass_larger_than_the_device(append):
     b.close()
 
 
+@pytest.mark.parametrize("groups", [False, True])
+@pytest.mark.parametrize("g,d", [(1, 128), (2, 64), (3, 128), (5, 64), (6, 128)])
+def test_decode_uncommon_head_ratios(g, d, groups):
+    """GQA ratios the benchmark's models do not use (MHA included): the split
+    pass's 4- and 8-row Q areas and the combine's head groups with columns
+    left unused.  Two shared prefixes, ragged private tails, requests outside
+    any group; every request against the oracle."""
+    need_gpu()
+    Hkv = 2
+    R = 14
+    group = [0, 0, 0, 0, 1, 1, 1, 1, 1, -1, -1, 0, 1, -1]
+    prefix_lens = [256, 512]
+    cached = [(prefix_lens[gi] if gi >= 0 else 0) + 1 + (53 * i) % 400 for i, gi in enumerate(group)]
+    w = make_workload("custom", seed=7 + g, custom=dict(Hq=g * Hkv, Hkv=Hkv, d=d, prefix_lens=prefix_lens,
+                                                      group=group, cached=cached, new=[1] * R,
+                                                      decode=[True] * R))
+    b = B.build_batch(w, poison=True)
+    out, lse = run_decode(b, use_groups=groups)
+    compare(b, out, lse, range(R))
+    b.close()
+
+
 def test_single_key_returns_value():
     """A context of one token returns that token's V (weight exactly 1)."""
     need_gpu()
