@@ -240,8 +240,8 @@ def test_grouped_members_need_not_be_contiguous():
     b.close()
 
 
-@pytest.mark.parametrize("append", [False, True])
-def test_prefix_pass_larger_than_the_device(append):
+@pytest.mark.parametrize("append,d", [(False, 128), (True, 128), (False, 64)])
+def test_prefix_pass_larger_than_the_device(append, d):
     """40 groups of 3 members over 8 kv heads: 320 shared-prefix CTAs (one key
     split each), three waves on a 152-SM device, so the split pass (launched
     once every prefix CTA has started, on all SMs) takes SMs only as
@@ -253,7 +253,7 @@ def test_prefix_pass_larger_than_the_device(append):
     group = [g for g in range(G) for _ in range(M)] + [-1] * 8
     cached = [(prefix_lens[g] if g >= 0 else 0) + 1 + (37 * i) % 300 for i, g in enumerate(group)]
     R = len(group)
-    w = make_workload("custom", custom=dict(Hq=32, Hkv=8, d=128, prefix_lens=prefix_lens, group=group,
+    w = make_workload("custom", custom=dict(Hq=32, Hkv=8, d=d, prefix_lens=prefix_lens, group=group,
                                           cached=cached, new=[1] * R, decode=[True] * R))
     b = B.build_batch(w, poison=True)
     out, lse = (run_decode_append if append else run_decode)(b, use_groups=True)
