@@ -605,101 +605,137 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (after_prefix) pdl_wait();
 }
 
-// Merge the partials of each (request, kv head) with log-sum-exp weights:
-// one warp per (request, kv head) merges the g q heads of that kv head, which
-// share one list of parts (the group's prefix splits, then the private
-// pieces).  Lane k holds part k's (m, l) for every head; lane c holds
-// elements [c*E, c*E + E) of every head's output.  All loads of a round are
-// in flight together.
-template <int D, int G>
-__global__ void __launch_bounds__(128) decode_combine_kernel(DecodeArgs a, DecodeLayout lay) {
-    constexpr int E = D / 32;   // output elements per lane and head
-    // G: q heads per kv head rounded up to 4 or 8 (g <= G)
+// Merge the partials of each (request, kv head) with log-sum-exp weights.
+// The g q heads of a kv head share one list of parts (the group's prefix
+// splits, then the private pieces); `wpi` warps split them, GW heads each.
+// Lane k holds part slot k's (m, l) for the warp's heads; lane c holds
+// elements [c*E, c*E + E) of every head's output.  With SPEC the partials of
+// slots 0 .. KR-1 are loaded in the same round as the part counts and the
+// (m, l): they are parts 0 .. KR-1 whenever the request's prefix partials
+// fill the prefix slots or number at least KR (every request of a one-group
+// batch), and are reloaded from their real slots otherwise; without it the
+// first round of partials waits for the counts like the others.
+template <int D, int GW, bool SPEC>
+__global__ void __launch_bounds__(128) decode_combine_kernel(DecodeArgs a, DecodeLayout lay, int32_t wpi) {
+    constexpr int E = D / 32;    // output elements per lane and head
+    constexpr int KR = 16 / GW;  // parts per round: KR x GW element vectors in flight per lane
     pdl_wait();
     const int lane = threadIdx.x & 31;
-    const int64_t item = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
+    const int64_t wid = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
+    const int64_t item = wpi == 2 ? wid >> 1 : wid;   // wpi is 1 or 2
     if (item >= (int64_t)lay.R * lay.Hkv) return;
     const int r = (int)(item / lay.Hkv), h = (int)(item % lay.Hkv);
     const int g = lay.g;
+    const int hs = wpi == 2 ? (int)(wid & 1) * GW : 0;   // the warp's first head within the kv head
+    const int ng = min(GW, g - hs);                // its heads (at least 1)
+    if (ng <= 0) return;
+    const int pph = lay.parts_per_head;
     const float *o_part = reinterpret_cast<const float *>(static_cast<const char *>(a.ws) + lay.off_o);
     const float2 *ml_part =
         reinterpret_cast<const float2 *>(static_cast<const char *>(a.ws) + lay.off_ml);
     const int32_t *nparts =
         reinterpret_cast<const int32_t *>(static_cast<const char *>(a.ws) + lay.off_nparts);
-    // The part counts written by the split pass (private pieces | prefix
-    // partials << 16) and, in the same round of loads, the (m, l) of every
-    // part slot: lane k holds slot k (prefix partials from 0, private pieces
-    // from prefix_parts); slots beyond the counts are masked once they are
-    // known (they may hold anything).
+    const int64_t head0 = (int64_t)r * lay.Hq + (int64_t)h * g + hs;   // (request, q head) index of head 0
+    auto load_part = [&](float (&dst)[E], int hd, int slot) {
+        const float *src = o_part + ((head0 + hd) * pph + slot) * D + lane * E;
+        if constexpr (E == 4) {
+            const float4 t = *reinterpret_cast<const float4 *>(src);
+            dst[0] = t.x; dst[1] = t.y; dst[2] = t.z; dst[3] = t.w;
+        } else {
+            const float2 t = *reinterpret_cast<const float2 *>(src);
+            dst[0] = t.x; dst[1] = t.y;
+        }
+    };
+    // one round: the part counts written by the split pass (private pieces
+    // | prefix partials << 16), the (m, l) of every part slot (lane k: slot
+    // k), and the partials of slots 0 .. KR-1; what lies beyond the counts
+    // may hold anything and is masked or replaced below
     const int32_t counts = nparts[item];
-    const int64_t head0 = (int64_t)r * lay.Hq + (int64_t)h * g;   // (request, q head) index of head 0
-    float2 mlv[G];
+    float2 mlv[GW];
 #pragma unroll
-    for (int hd = 0; hd < G; ++hd) {
+    for (int hd = 0; hd < GW; ++hd) {
         mlv[hd] = make_float2(-INFINITY, 0.f);
-        if (hd < g && lane < lay.parts_per_head) mlv[hd] = ml_part[(head0 + hd) * lay.parts_per_head + lane];
+        if (hd < ng && lane < pph) mlv[hd] = ml_part[(head0 + hd) * pph + lane];
     }
-    const int n_priv = min(max(counts & 0xFFFF, 0), kMaxPrivateParts);
+    float v[KR][GW][E];
+#pragma unroll
+    for (int u = 0; u < KR; ++u)
+#pragma unroll
+        for (int hd = 0; hd < GW; ++hd) {
+#pragma unroll
+            for (int e = 0; e < E; ++e) v[u][hd][e] = 0.f;
+            if (SPEC && hd < ng && u < pph) load_part(v[u][hd], hd, u);
+        }
+    const int n_priv = min(max(counts & 0xFFFF, 0), pph - lay.prefix_parts);
     const int n_pre = min((counts >> 16) & 0xFFFF, lay.prefix_parts);
     const int total = min(n_pre + n_priv, 32);
     const bool live = lane < n_pre || (lane >= lay.prefix_parts && lane < lay.prefix_parts + n_priv);
     // parts in merge order: the prefix partials, then the private pieces
     auto part_lane = [&](int k) { return k < n_pre ? k : lay.prefix_parts + (k - n_pre); };
-    auto part_slot = [&](int hd, int k) { return (head0 + hd) * lay.parts_per_head + part_lane(k); };
     // weights: the lane of a slot owns that slot's weight for every head
-    float wk[G], mx[G], den[G];
+    float wk[GW], mx[GW], den[GW];
 #pragma unroll
-    for (int hd = 0; hd < G; ++hd) {
-        mx[hd] = (hd < g && live) ? mlv[hd].x : -INFINITY;
+    for (int hd = 0; hd < GW; ++hd) {
+        mx[hd] = (hd < ng && live) ? mlv[hd].x : -INFINITY;
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) mx[hd] = fmaxf(mx[hd], __shfl_xor_sync(0xffffffffu, mx[hd], off));
     }
 #pragma unroll
-    for (int hd = 0; hd < G; ++hd) {
-        const float w = (hd < g && live) ? fast_exp2(mlv[hd].x - mx[hd]) : 0.f;
-        den[hd] = (hd < g && live) ? w * mlv[hd].y : 0.f;
+    for (int hd = 0; hd < GW; ++hd) {
+        const float w = (hd < ng && live) ? fast_exp2(mlv[hd].x - mx[hd]) : 0.f;
+        den[hd] = (hd < ng && live) ? w * mlv[hd].y : 0.f;
         wk[hd] = w;
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) den[hd] += __shfl_xor_sync(0xffffffffu, den[hd], off);
     }
-    float acc[G][E];
+    float acc[GW][E];
 #pragma unroll
-    for (int hd = 0; hd < G; ++hd)
+    for (int hd = 0; hd < GW; ++hd)
 #pragma unroll
         for (int e = 0; e < E; ++e) acc[hd][e] = 0.f;
-    // parts in rounds of KR (KR x G element vectors in flight per lane)
-    constexpr int KR = 16 / G;
-    for (int k0 = 0; k0 < total; k0 += KR) {
-        float v[KR][G][E];
+    // the first round: keep what was loaded where part u sits in slot u,
+    // reload it where it does not, and drop slots past the parts
+#pragma unroll
+    for (int u = 0; u < KR; ++u)
+#pragma unroll
+        for (int hd = 0; hd < GW; ++hd) {
+            if (u >= total) {
+#pragma unroll
+                for (int e = 0; e < E; ++e) v[u][hd][e] = 0.f;
+            } else if ((!SPEC || part_lane(u) != u) && hd < ng) {
+                load_part(v[u][hd], hd, part_lane(u));
+            }
+        }
+#pragma unroll
+    for (int u = 0; u < KR; ++u)
+#pragma unroll
+        for (int hd = 0; hd < GW; ++hd) {
+            const float w = __shfl_sync(0xffffffffu, wk[hd], u < total ? part_lane(u) : 0);
+#pragma unroll
+            for (int e = 0; e < E; ++e) acc[hd][e] += w * v[u][hd][e];
+        }
+    // the other parts in rounds of KR
+    for (int k0 = KR; k0 < total; k0 += KR) {
 #pragma unroll
         for (int u = 0; u < KR; ++u)
 #pragma unroll
-            for (int hd = 0; hd < G; ++hd) {
+            for (int hd = 0; hd < GW; ++hd) {
 #pragma unroll
                 for (int e = 0; e < E; ++e) v[u][hd][e] = 0.f;
-                if (k0 + u < total && hd < g) {
-                    const float *src = o_part + part_slot(hd, k0 + u) * D + lane * E;
-                    if constexpr (E == 4) {
-                        const float4 t = *reinterpret_cast<const float4 *>(src);
-                        v[u][hd][0] = t.x; v[u][hd][1] = t.y; v[u][hd][2] = t.z; v[u][hd][3] = t.w;
-                    } else {
-                        const float2 t = *reinterpret_cast<const float2 *>(src);
-                        v[u][hd][0] = t.x; v[u][hd][1] = t.y;
-                    }
-                }
+                if (k0 + u < total && hd < ng) load_part(v[u][hd], hd, part_lane(k0 + u));
             }
 #pragma unroll
         for (int u = 0; u < KR; ++u)
 #pragma unroll
-            for (int hd = 0; hd < G; ++hd) {
+            for (int hd = 0; hd < GW; ++hd) {
                 const float w = __shfl_sync(0xffffffffu, wk[hd], k0 + u < total ? part_lane(k0 + u) : 0);
 #pragma unroll
                 for (int e = 0; e < E; ++e) acc[hd][e] += w * v[u][hd][e];
             }
     }
 #pragma unroll
-    for (int hd = 0; hd < G; ++hd) {
-        if (hd >= g) break;
+    for (int hd = 0; hd < GW; ++hd) {
+        if (hd >= ng) break;
         const float inv = 1.f / den[hd];
         uint16_t *out = static_cast<uint16_t *>(a.out) + (head0 + hd) * D + lane * E;
         if constexpr (E == 4) {
@@ -852,14 +888,25 @@ static cudaError_t launch_decode_t(const DecodeLayout &L, const DecodeArgs &a, i
 
 template <int D>
 static cudaError_t launch_combine_t(const DecodeLayout &L, const DecodeArgs &a, cudaStream_t stream, Tracer *tr) {
-    // four warps per CTA: small batches spread over more SMs
-    const int64_t items = (int64_t)L.R * L.Hkv;
-    const int64_t cgrid = (items + 3) / 4;
+    // Four warps per CTA.  While the (request, kv head) items alone would
+    // leave the device's warps idle (at most 8 items per SM), each item's
+    // heads are split over two warps of 2 (g <= 4) or 4 heads, which keep 8
+    // or 4 parts in flight per round, the first round loaded with the part
+    // counts (measured on the Qwen2.5-7B mixed batch, 1024 items: decode
+    // 89.3 -> 88.2 us); with more items one warp takes every head (the
+    // split and the early round measured slower on 4096-item batches).
+    const bool split = (int64_t)L.R * L.Hkv <= 8LL * L.sms;
+    const int gw = split ? (L.g <= 4 ? 2 : 4) : (L.g <= 4 ? 4 : 8);
+    const int32_t wpi = (L.g + gw - 1) / gw;   // 1 or 2 (g <= 8)
+    const int64_t warps = (int64_t)L.R * L.Hkv * wpi;
+    const int64_t cgrid = (warps + 3) / 4;
     if (cgrid > 0x7fffffff) return cudaErrorInvalidConfiguration;
     if (tr) tr->begin(kKernelDecodeCombine, stream);
-    cudaError_t e = L.g <= 4
-                        ? launch_pdl(decode_combine_kernel<D, 4>, dim3((unsigned)cgrid), dim3(128), 0, stream, a, L)
-                        : launch_pdl(decode_combine_kernel<D, 8>, dim3((unsigned)cgrid), dim3(128), 0, stream, a, L);
+    const dim3 cg((unsigned)cgrid), cb(128);
+    cudaError_t e = gw == 2   ? launch_pdl(decode_combine_kernel<D, 2, true>, cg, cb, 0, stream, a, L, wpi)
+                    : split   ? launch_pdl(decode_combine_kernel<D, 4, true>, cg, cb, 0, stream, a, L, wpi)
+                    : gw == 4 ? launch_pdl(decode_combine_kernel<D, 4, false>, cg, cb, 0, stream, a, L, wpi)
+                              : launch_pdl(decode_combine_kernel<D, 8, false>, cg, cb, 0, stream, a, L, wpi);
     if (tr) tr->end(kKernelDecodeCombine, stream);
     return e;
 }
